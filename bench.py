@@ -1,0 +1,385 @@
+"""Benchmark of the DO-loss forward+backward path on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+A step is one do_forward_backward call (Top-K signatures, Hamming matrix,
+loss and dlogits) over the E=128, k=8, T=65536 router-logit workload (the
+30BA3B-shaped layer).  Inputs are resident in HBM when the timed region
+starts; consecutive steps rotate over 8 buffer sets (about 520 MiB, four times
+the L2) so no step reads what the previous one left in L2.  Rank 0 prints one
+JSON line.  With N > 1 (torchrun, one process per GPU) every rank runs an
+independent replica: the path has no exchange step on one window, so the job
+is weak-scaled replicas and the value is the tokens of all ranks over the
+slowest rank's time.
+
+--impl reference times the CPU oracle (the only reference this method has:
+the paper publishes no code) on the host cores, on a bounded token sample of
+the same workload per step.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+WORKLOAD = "c3"
+METRIC = "DO-loss fwd+bwd routed tokens/s at E=128,k=8; % of GB300 HBM roofline"
+UNIT = "tokens/s"
+N_SETS = 8
+KERNELS_PER_STEP = 4  # signatures, pairwise Hamming, loss, loss finalize
+
+
+def algorithmic_bytes(T, E, L=1):
+    """Bytes the path must move once: logits read and dlogits written (4TE
+    each), signatures written and read back (2 x 4EW), the Hamming matrix
+    written and read (2 x 4E^2) and the counts (4E) -- per problem."""
+    W = (T + 31) // 32
+    return L * (8 * T * E + 8 * E * W + 8 * E * E + 4 * E)
+
+
+def stage_bytes(T, E, L=1):
+    W = (T + 31) // 32
+    return {
+        "signatures": L * (4 * T * E + 4 * E * W + 4 * E),
+        "pairwise_hamming": L * (4 * E * W + 4 * E * E),
+        "loss_fwd_bwd": L * (4 * T * E + 4 * E * W + 4 * E * E + 4 * T * E),
+    }
+
+
+def measured_peaks():
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except Exception:
+        return None
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2609_32398_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        h.update(open(os.path.join(csrc, f), "rb").read())
+    return h.hexdigest()[:12]
+
+
+def profiled_traffic(stage):
+    """DRAM bytes per launch of `stage` from the committed ncu summary, if it was
+    captured on the current kernel sources (else None)."""
+    path = os.path.join(ROOT, "profiles", "traffic.md")
+    if not os.path.exists(path):
+        return None
+    src = kernel_source_hash()
+    for line in open(path):
+        m = re.match(r"\|\s*(\w+)\s*\|\s*([0-9a-f]{12})\s*\|\s*(\d+)\s*\|", line)
+        if m and m.group(1) == stage and m.group(2) == src:
+            return int(m.group(3))
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi samples (every 200 ms) of SM clock and throttle reasons."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_setup(gpus):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl")
+    return rank, world, local
+
+
+def reduce_max(x: float, world: int, device) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+
+
+def oracle_throughput(z_np, k, gate, budget_s, max_tokens=None):
+    """Oracle forward+backward over leading token samples of z until `budget_s`
+    seconds have been spent; returns (tokens/s, tokens, seconds, runs)."""
+    import oracle
+
+    T = z_np.shape[0]
+    n = T if max_tokens is None else min(T, max_tokens)
+    tokens, spent, runs = 0, 0.0, 0
+    while runs == 0 or spent < budget_s:
+        t0 = time.perf_counter()
+        oracle.forward_backward(z_np[:n], k, gate)
+        spent += time.perf_counter() - t0
+        tokens += n
+        runs += 1
+    return tokens / spent, tokens, spent, runs
+
+
+def run_reference(args, rank, world):
+    """The reference arm: the CPU oracle as it stands, on the host cores."""
+    import numpy as np
+
+    from paper_2609_32398_gb300 import workloads
+
+    if rank != 0:
+        return
+    w = workloads.get(WORKLOAD)
+    import oracle
+
+    oracle.build()
+    z = np.ascontiguousarray(workloads.logits(w, "cpu")[0].numpy())
+    # Calibrate a per-step token sample so that warmup + steps take about two minutes.
+    t0 = time.perf_counter()
+    oracle.forward_backward(z[:2048], w.k, w.gate)
+    per_tok = (time.perf_counter() - t0) / 2048
+    steps = args.steps + args.warmup
+    sample = int(max(256, min(w.T, 120.0 / max(1, steps) / per_tok)))
+    sample -= sample % 32 if sample > 32 else 0
+    for i in range(args.warmup):
+        oracle.forward_backward(z[:sample], w.k, w.gate)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        oracle.forward_backward(z[:sample], w.k, w.gate)
+    dt = time.perf_counter() - t0
+    value = sample * args.steps / dt
+    desc = (f"leading {sample} of the {w.T} tokens of the E=128 k=8 workload per step, "
+            f"single-threaded C oracle in double precision")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": config_dict(w),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def config_dict(w):
+    return {"workload": f"3B-active-shaped router layer: E={w.E} k={w.k} T={w.T} L={w.L}",
+            "E": w.E, "k": w.k, "T": w.T, "L": w.L, "gate": "sigmoid_norm",
+            "l2": f"{N_SETS} rotating buffer sets (~{N_SETS * algorithmic_bytes(w.T, w.E) // 2**20} MiB) > L2",
+            "parallelism": "replicas"}
+
+
+def run_ours(args, rank, world, local):
+    import numpy as np
+    import torch
+
+    import paper_2609_32398_gb300.doloss as dl
+    from paper_2609_32398_gb300 import workloads
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    dl.lib()
+    w = workloads.get(WORKLOAD)
+    T, E, k, L = w.T, w.E, w.k, w.L
+    base = workloads.logits(w, dev)
+    sets = []
+    for s in range(N_SETS):
+        z = base if s == 0 else (base + 0.0)   # same values, distinct HBM buffers
+        sets.append((z, dl.Buffers(L, T, E, k, dev)))
+    stream = torch.cuda.current_stream(dev)
+
+    def step(i):
+        z, out = sets[i % N_SETS]
+        dl.forward_backward(z, k, w.gate, 1.0, out=out)
+
+    warm = max(3, args.warmup)
+    sampler = ClockSampler(local)
+    sampler.start()
+    for i in range(warm):
+        step(i)
+    torch.cuda.synchronize()
+    # untimed soak so the clocks reach their loaded state and get sampled
+    t_soak = time.perf_counter()
+    i = 0
+    while time.perf_counter() - t_soak < 1.0:
+        step(i)
+        i += 1
+        if i % 256 == 0:
+            torch.cuda.synchronize()
+    torch.cuda.synchronize()
+
+    barrier(world)
+    torch.cuda.synchronize()
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for i in range(args.steps):
+        step(i)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    clocks = sampler.stop()
+    ms = ev0.elapsed_time(ev1)
+    ms_max = reduce_max(ms, world, dev)
+    ms_per_step = ms_max / args.steps
+    value = world * T * L / (ms_per_step * 1e-3)
+
+    st = dl.device_status(sets[0][1].workspace)
+    if st != 0:
+        raise RuntimeError(f"device status after the timed region: {dl.status_string(st)}")
+
+    # Per-stage durations: the same launches through the split entry points,
+    # with events between them on the launching stream.
+    stage_ms = {"signatures": 0.0, "pairwise_hamming": 0.0, "loss_fwd_bwd": 0.0}
+    reps = max(20, min(args.steps, 2000))
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(4 * reps)]
+    for r in range(reps):
+        z, out = sets[r % N_SETS]
+        e = evs[4 * r:4 * r + 4]
+        e[0].record(stream)
+        dl.signatures(z, k, out.bits, out.counts)
+        e[1].record(stream)
+        dl.pairwise_hamming(out.bits, T, out.D)
+        e[2].record(stream)
+        dl.loss_fwd_bwd(z, out.bits, out.D, k, w.gate, workspace=out.workspace, dlogits=out.dlogits)
+        e[3].record(stream)
+    torch.cuda.synchronize()
+    for r in range(reps):
+        e = evs[4 * r:4 * r + 4]
+        stage_ms["signatures"] += e[0].elapsed_time(e[1]) / reps
+        stage_ms["pairwise_hamming"] += e[1].elapsed_time(e[2]) / reps
+        stage_ms["loss_fwd_bwd"] += e[2].elapsed_time(e[3]) / reps
+    dom = max(stage_ms, key=stage_ms.get)
+    peaks = measured_peaks()
+    peak = peaks["hbm_gbs"] if peaks else 6800.0
+    peak_src = "of measured" if peaks else "of fallback"
+    sb = stage_bytes(T, E, L)
+    achieved = sb[dom] / (stage_ms[dom] * 1e-3) / 1e9
+    step_gbs = algorithmic_bytes(T, E, L) / (ms_per_step * 1e-3) / 1e9
+
+    # End to end through the host entry point: pinned logits in, dlogits and loss out.
+    e2e = None
+    if rank == 0 or world > 1:
+        hz = base.cpu().pin_memory()
+        hdz = torch.empty_like(hz).pin_memory()
+        hloss = torch.empty(L, dtype=torch.float32).pin_memory()
+        dbuf = torch.empty(dl.host_buffer_size(T, E, k, L), dtype=torch.uint8, device=dev)
+        for _ in range(3):
+            dl.forward_backward_host(hz, k, w.gate, device_buffer=dbuf, h_dlogits=hdz, h_loss=hloss)
+        n_e2e = max(3, min(args.steps, 50))
+        barrier(world)
+        t0 = time.perf_counter()
+        for _ in range(n_e2e):
+            dl.forward_backward_host(hz, k, w.gate, device_buffer=dbuf, h_dlogits=hdz, h_loss=hloss)
+        dt = reduce_max((time.perf_counter() - t0) / n_e2e, world, dev)
+        e2e = {"value": world * T * L / dt, "unit": UNIT, "h2d_bytes_per_step": 4 * T * E * L,
+               "d2h_bytes_per_step": 4 * T * E * L + 4 * L, "ms_per_step": dt * 1e3}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        zc = np.ascontiguousarray(base[0].cpu().numpy())
+        rate, ntok, spent, runs = oracle_throughput(zc, k, w.gate, budget_s=10.0)
+        cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
+               "sample": f"{runs} oracle run(s) over all {T} tokens of the same workload "
+                         f"({spent:.1f} s, single-threaded C, double precision)"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": warm, "ms_per_step": ms_per_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": config_dict(w),
+            "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak,
+                         "unit": "GB/s", "frac": achieved / peak, "peak_source": peak_src,
+                         "traffic": profiled_traffic(dom),
+                         "stage_us": {k_: v * 1e3 for k_, v in stage_ms.items()}},
+            "roofline_step": {"achieved": step_gbs, "peak": peak, "unit": "GB/s",
+                              "frac": step_gbs / peak, "bytes_per_step": algorithmic_bytes(T, E, L)},
+            "clocks": clocks, "e2e": e2e, "gpu_launches": KERNELS_PER_STEP * args.steps,
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        rank = int(os.environ.get("RANK", "0"))
+        world = int(os.environ.get("WORLD_SIZE", str(args.gpus)))
+        run_reference(args, rank, world)
+        return
+    rank, world, local = dist_setup(args.gpus)
+    try:
+        run_ours(args, rank, world, local)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

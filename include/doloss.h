@@ -1,0 +1,141 @@
+/*
+ * doloss.h -- C ABI of the GB300 DO-loss library (libdoloss.so).
+ *
+ * The Distributional Orthogonalization loss of "Function Over Form:
+ * Distributional Orthogonalization in Mixture-of-Experts with Replica Expert
+ * Mechanism" on one GPU, as four steps:
+ *   1. Top-K routing of T tokens over E experts, packed into binary load
+ *      signatures with per-expert counts               (Sec. 3.1.1, Eq. 1)
+ *   2. the all-pairs Hamming matrix of the signatures  (Sec. 3.1.3, Eq. gij_cij)
+ *   3. the surrogate loss and its gradient to the router logits
+ *                                                       (Sec. 3.1.3, Eq. do_loss)
+ *   4. Eq. origin_do, the sum of squared distances, as a diagnostic.
+ *
+ * Notation: E experts (the paper's n), k selected per token (K), T tokens in
+ * the signature window (m), L independent problems batched in one call (for
+ * example the MoE layers of a model), W = ceil(T/32).
+ *
+ * Conventions shared by every entry point:
+ *  - Every array argument is a DEVICE pointer owned by the caller, except in
+ *    do_forward_backward_host, whose h_* arguments are host pointers.  The
+ *    library allocates nothing and keeps no state between calls.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default
+ *    stream).  Calls are asynchronous on it, except do_device_status and
+ *    do_forward_backward_host, which synchronize it.
+ *  - Arguments are validated before anything is launched; a rejected call
+ *    returns DO_ERR_INVALID_ARG or DO_ERR_UNSUPPORTED and touches no memory.
+ *    A failed launch returns DO_ERR_CUDA.  Conditions only the device can see
+ *    (a Hamming row sum that does not fit int32, a device wait that ran out)
+ *    are recorded in the workspace and reported by do_device_status.
+ *  - Layouts are dense and row-major:
+ *      logits, dlogits  [L][T][E] fp32 (token-major: one row per token)
+ *      bits             [L][E][W] uint32; bit (t mod 32) of word t/32 of row i
+ *                       is f_it; bits of positions t >= T are zero
+ *      counts           [L][E]    int32, n_i = ||F_i||_1
+ *      D                [L][E][E] int32, D_ij = ||F_i - F_j||_1 (symmetric,
+ *                       zero diagonal)
+ *      loss             [L] fp32; origin_do [L] int64
+ *  - Logits must be finite.  Top-K is taken on the raw logits: larger value
+ *    first, equal values in favour of the lower expert index (the gates are
+ *    monotone, so this is the Top-K of the gated scores).
+ *  - Limits: 1 <= k <= E <= 1024, T >= 1, L >= 1, (E-1)*T < 2^31.  float
+ *    arrays need 4-byte alignment (16-byte alignment and E % 4 == 0 select
+ *    the vectorised kernels); uint32/int32 arrays 4-byte, int64 8-byte.
+ *  - Results are deterministic: bits, counts, D and origin_do are exact
+ *    integers; loss and dlogits are bitwise reproducible run to run (fixed
+ *    reduction order, no floating-point atomics).
+ */
+#ifndef DOLOSS_H
+#define DOLOSS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    DO_OK = 0,
+    DO_ERR_INVALID_ARG = 1,  /* null pointer, bad size or alignment          */
+    DO_ERR_UNSUPPORTED = 2,  /* valid but outside this build's limits        */
+    DO_ERR_CUDA = 3,         /* a CUDA runtime call or launch failed         */
+    DO_ERR_TIMEOUT = 4,      /* a bounded device wait ran out                */
+    DO_ERR_OVERFLOW = 5,     /* a row sum of D does not fit int32            */
+    DO_ERR_WORKSPACE = 6     /* workspace missing or smaller than required   */
+} do_status;
+
+typedef enum {
+    DO_GATE_SIGMOID_NORM = 0, /* s = sigmoid(z), p = s / sum(s)  (Sec. 3.1.1, App. A) */
+    DO_GATE_SOFTMAX = 1       /* p = softmax(z)                                        */
+} do_gate;
+
+/* Step 1 (Sec. 3.1.1, Eq. 1: f_it = 1(i in Top-K(x_t))).
+ * Reads logits [L][T][E]; writes the load signatures bits [L][E][W] and the
+ * per-expert token counts [L][E] (written, not accumulated). */
+do_status do_signatures(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
+                        uint32_t *bits, int32_t *counts, void *stream);
+
+/* Step 2 (Sec. 3.1.3, Eq. gij_cij: G_ij = ||F_i - F_j||_1).
+ * Reads bits [L][E][W]; writes D [L][E][E], the exact number of tokens on
+ * which experts i and j disagree. */
+do_status do_pairwise_hamming(const uint32_t *bits, int64_t T, int32_t E, int32_t L,
+                              int32_t *D, void *stream);
+
+/* Step 3 (Sec. 3.1.3, Eq. do_loss; Sec. 3.1.4, Eq. global_do):
+ *   L_DO = 1/(T^2 k) sum_i sum_j G_ij C_ij,  C_ij = sum_t p_it (f_it - f_jt),
+ * with G = d_scale * D held constant (detached) and p the dense router
+ * probability of `gate`.  d_scale is 1 for a local matrix, or 1/|replicas|
+ * when D is the sum of the replicas' matrices (Global-DO).
+ * Writes loss [L] (unscaled by grad_scale), origin_do [L] = sum_{i!=j} D_ij^2
+ * (Eq. origin_do; may be NULL) and dlogits [L][T][E] = grad_scale * dL/dz
+ * (may be NULL for a forward-only call).  bits must hold the selection that
+ * produced the token rows of logits; D may come from any source whose row
+ * sums fit int32.  workspace: do_workspace_size(T, E, k, L) bytes of device
+ * memory, 256-byte aligned, reused across calls; its contents need no
+ * initialisation. */
+do_status do_loss_fwd_bwd(const float *logits, const uint32_t *bits, const int32_t *D,
+                          int64_t T, int32_t E, int32_t k, int32_t L, int32_t gate,
+                          float d_scale, float grad_scale, float *loss, int64_t *origin_do,
+                          float *dlogits, void *workspace, size_t workspace_bytes,
+                          void *stream);
+
+/* Steps 1-3 in one call on a local window (d_scale = 1): logits in; bits,
+ * counts, D, loss, origin_do (may be NULL) and dlogits (may be NULL) out. */
+do_status do_forward_backward(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
+                              int32_t gate, float grad_scale, uint32_t *bits, int32_t *counts,
+                              int32_t *D, float *loss, int64_t *origin_do, float *dlogits,
+                              void *workspace, size_t workspace_bytes, void *stream);
+
+/* Device workspace, in bytes, that do_loss_fwd_bwd and do_forward_backward
+ * need for these sizes (0 if the sizes are invalid). */
+size_t do_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L);
+
+/* Synchronizes `stream`, then reads and clears the device-side status that
+ * the previous calls with this workspace recorded: DO_OK, DO_ERR_OVERFLOW or
+ * DO_ERR_TIMEOUT (outputs of the failing call are then undefined). */
+do_status do_device_status(void *workspace, void *stream);
+
+/* Host-to-host convenience over do_forward_backward: copies h_logits [L][T][E]
+ * to the device, runs steps 1-3, and copies loss [L] into h_loss and, when
+ * given, dlogits into h_dlogits [L][T][E], counts into h_counts [L][E] and D
+ * into h_D [L][E][E].  All device memory comes from `device_buffer`
+ * (do_host_buffer_size(T, E, k, L) bytes, 256-byte aligned).  Synchronous:
+ * returns after the results are in host memory and the device status has been
+ * checked.  Pinned host memory gives the full copy bandwidth. */
+do_status do_forward_backward_host(const float *h_logits, int64_t T, int32_t E, int32_t k,
+                                   int32_t L, int32_t gate, float grad_scale, float *h_loss,
+                                   float *h_dlogits, int32_t *h_counts, int32_t *h_D,
+                                   void *device_buffer, size_t device_buffer_bytes,
+                                   void *stream);
+
+size_t do_host_buffer_size(int64_t T, int32_t E, int32_t k, int32_t L);
+
+/* A static description of a status code. */
+const char *do_status_string(int32_t status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DOLOSS_H */

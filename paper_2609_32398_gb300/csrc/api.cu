@@ -1,0 +1,202 @@
+// C ABI of libdoloss (declared in include/doloss.h): argument validation,
+// workspace layout and the launch sequence of each entry point.
+#include <cuda_runtime.h>
+
+#include <climits>
+#include <cstdint>
+
+#include "dol_internal.cuh"
+#include "doloss.h"
+
+namespace {
+
+using dol::Problem;
+
+bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+do_status check_sizes(int64_t T, int32_t E, int32_t k, int32_t L, Problem *p) {
+    if (T < 1 || E < 1 || k < 1 || k > E || L < 1) return DO_ERR_INVALID_ARG;
+    if (E > 1024 || L > 65535) return DO_ERR_UNSUPPORTED;
+    if ((int64_t)(E - 1) * T > (int64_t)INT_MAX) return DO_ERR_UNSUPPORTED;
+    p->T = T;
+    p->E = E;
+    p->k = k;
+    p->L = L;
+    p->W = (T + 31) / 32;
+    return DO_OK;
+}
+
+do_status from_cuda(cudaError_t e) { return e == cudaSuccess ? DO_OK : DO_ERR_CUDA; }
+
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Device buffer of do_forward_backward_host, carved in this order.
+struct HostBufLayout {
+    size_t logits, bits, counts, D, loss, dlogits, ws, total;
+};
+
+HostBufLayout host_layout(const Problem &p) {
+    HostBufLayout b;
+    size_t off = 0;
+    const size_t te = (size_t)p.L * (size_t)p.T * (size_t)p.E;
+    b.logits = off; off = round_up(off + sizeof(float) * te, 256);
+    b.bits = off;   off = round_up(off + sizeof(uint32_t) * (size_t)p.L * p.E * p.W, 256);
+    b.counts = off; off = round_up(off + sizeof(int32_t) * (size_t)p.L * p.E, 256);
+    b.D = off;      off = round_up(off + sizeof(int32_t) * (size_t)p.L * p.E * p.E, 256);
+    b.loss = off;   off = round_up(off + sizeof(float) * (size_t)p.L, 256);
+    b.dlogits = off; off = round_up(off + sizeof(float) * te, 256);
+    b.ws = off;     off = round_up(off + dol::workspace_bytes(p), 256);
+    b.total = off;
+    return b;
+}
+
+}  // namespace
+
+extern "C" {
+
+do_status do_signatures(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
+                        uint32_t *bits, int32_t *counts, void *stream) {
+    Problem p;
+    do_status st = check_sizes(T, E, k, L, &p);
+    if (st != DO_OK) return st;
+    if (!logits || !bits || !counts) return DO_ERR_INVALID_ARG;
+    if (!aligned(logits, 4) || !aligned(bits, 4) || !aligned(counts, 4)) return DO_ERR_INVALID_ARG;
+    return from_cuda(dol::launch_signatures(logits, p, bits, counts, (cudaStream_t)stream));
+}
+
+do_status do_pairwise_hamming(const uint32_t *bits, int64_t T, int32_t E, int32_t L, int32_t *D,
+                              void *stream) {
+    Problem p;
+    do_status st = check_sizes(T, E, 1, L, &p);
+    if (st != DO_OK) return st;
+    if (!bits || !D) return DO_ERR_INVALID_ARG;
+    if (!aligned(bits, 4) || !aligned(D, 4)) return DO_ERR_INVALID_ARG;
+    return from_cuda(dol::launch_hamming(bits, p, D, (cudaStream_t)stream));
+}
+
+do_status do_loss_fwd_bwd(const float *logits, const uint32_t *bits, const int32_t *D, int64_t T,
+                          int32_t E, int32_t k, int32_t L, int32_t gate, float d_scale,
+                          float grad_scale, float *loss, int64_t *origin_do, float *dlogits,
+                          void *workspace, size_t workspace_bytes, void *stream) {
+    Problem p;
+    do_status st = check_sizes(T, E, k, L, &p);
+    if (st != DO_OK) return st;
+    if (!logits || !bits || !D || !loss) return DO_ERR_INVALID_ARG;
+    if (gate != DO_GATE_SIGMOID_NORM && gate != DO_GATE_SOFTMAX) return DO_ERR_INVALID_ARG;
+    if (!(d_scale == d_scale) || !(grad_scale == grad_scale)) return DO_ERR_INVALID_ARG;
+    if (!aligned(logits, 4) || !aligned(bits, 4) || !aligned(D, 4) || !aligned(loss, 4) ||
+        (dlogits && !aligned(dlogits, 4)) || (origin_do && !aligned(origin_do, 8)))
+        return DO_ERR_INVALID_ARG;
+    if (!workspace || !aligned(workspace, 256) || workspace_bytes < dol::workspace_bytes(p))
+        return DO_ERR_WORKSPACE;
+    return from_cuda(dol::launch_loss(logits, bits, D, p, gate, d_scale, grad_scale, loss,
+                                      reinterpret_cast<long long *>(origin_do), dlogits,
+                                      workspace, (cudaStream_t)stream));
+}
+
+do_status do_forward_backward(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
+                              int32_t gate, float grad_scale, uint32_t *bits, int32_t *counts,
+                              int32_t *D, float *loss, int64_t *origin_do, float *dlogits,
+                              void *workspace, size_t workspace_bytes, void *stream) {
+    Problem p;
+    do_status st = check_sizes(T, E, k, L, &p);
+    if (st != DO_OK) return st;
+    if (!logits || !bits || !counts || !D || !loss) return DO_ERR_INVALID_ARG;
+    if (gate != DO_GATE_SIGMOID_NORM && gate != DO_GATE_SOFTMAX) return DO_ERR_INVALID_ARG;
+    if (!(grad_scale == grad_scale)) return DO_ERR_INVALID_ARG;
+    if (!aligned(logits, 4) || !aligned(bits, 4) || !aligned(counts, 4) || !aligned(D, 4) ||
+        !aligned(loss, 4) || (dlogits && !aligned(dlogits, 4)) ||
+        (origin_do && !aligned(origin_do, 8)))
+        return DO_ERR_INVALID_ARG;
+    if (!workspace || !aligned(workspace, 256) || workspace_bytes < dol::workspace_bytes(p))
+        return DO_ERR_WORKSPACE;
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaError_t e = dol::launch_signatures(logits, p, bits, counts, s);
+    if (e == cudaSuccess) e = dol::launch_hamming(bits, p, D, s);
+    if (e == cudaSuccess)
+        e = dol::launch_loss(logits, bits, D, p, gate, 1.0f, grad_scale, loss,
+                             reinterpret_cast<long long *>(origin_do), dlogits, workspace, s);
+    return from_cuda(e);
+}
+
+size_t do_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L) {
+    Problem p;
+    if (check_sizes(T, E, k, L, &p) != DO_OK) return 0;
+    return dol::workspace_bytes(p);
+}
+
+do_status do_device_status(void *workspace, void *stream) {
+    if (!workspace || !aligned(workspace, 256)) return DO_ERR_WORKSPACE;
+    cudaStream_t s = (cudaStream_t)stream;
+    int flags = 0;
+    cudaError_t e = cudaMemcpyAsync(&flags, workspace, sizeof(int), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(workspace, 0, sizeof(int), s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return DO_ERR_CUDA;
+    if (flags & dol::kDevTimeout) return DO_ERR_TIMEOUT;
+    if (flags & dol::kDevOverflow) return DO_ERR_OVERFLOW;
+    return DO_OK;
+}
+
+size_t do_host_buffer_size(int64_t T, int32_t E, int32_t k, int32_t L) {
+    Problem p;
+    if (check_sizes(T, E, k, L, &p) != DO_OK) return 0;
+    return host_layout(p).total;
+}
+
+do_status do_forward_backward_host(const float *h_logits, int64_t T, int32_t E, int32_t k,
+                                   int32_t L, int32_t gate, float grad_scale, float *h_loss,
+                                   float *h_dlogits, int32_t *h_counts, int32_t *h_D,
+                                   void *device_buffer, size_t device_buffer_bytes, void *stream) {
+    Problem p;
+    do_status st = check_sizes(T, E, k, L, &p);
+    if (st != DO_OK) return st;
+    if (!h_logits || !h_loss) return DO_ERR_INVALID_ARG;
+    const HostBufLayout b = host_layout(p);
+    if (!device_buffer || !aligned(device_buffer, 256) || device_buffer_bytes < b.total)
+        return DO_ERR_WORKSPACE;
+    char *base = static_cast<char *>(device_buffer);
+    float *d_logits = reinterpret_cast<float *>(base + b.logits);
+    uint32_t *d_bits = reinterpret_cast<uint32_t *>(base + b.bits);
+    int32_t *d_counts = reinterpret_cast<int32_t *>(base + b.counts);
+    int32_t *d_D = reinterpret_cast<int32_t *>(base + b.D);
+    float *d_loss = reinterpret_cast<float *>(base + b.loss);
+    float *d_dlogits = h_dlogits ? reinterpret_cast<float *>(base + b.dlogits) : nullptr;
+    void *ws = base + b.ws;
+    cudaStream_t s = (cudaStream_t)stream;
+    const size_t te = sizeof(float) * (size_t)p.L * p.T * p.E;
+
+    // A cleared status word, so that do_device_status below sees this call only.
+    cudaError_t e = cudaMemsetAsync(ws, 0, sizeof(int), s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(d_logits, h_logits, te, cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return DO_ERR_CUDA;
+    st = do_forward_backward(d_logits, T, E, k, L, gate, grad_scale, d_bits, d_counts, d_D, d_loss,
+                             nullptr, d_dlogits, ws, dol::workspace_bytes(p), stream);
+    if (st != DO_OK) return st;
+    e = cudaMemcpyAsync(h_loss, d_loss, sizeof(float) * p.L, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess && h_dlogits)
+        e = cudaMemcpyAsync(h_dlogits, d_dlogits, te, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess && h_counts)
+        e = cudaMemcpyAsync(h_counts, d_counts, sizeof(int32_t) * (size_t)p.L * p.E,
+                            cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess && h_D)
+        e = cudaMemcpyAsync(h_D, d_D, sizeof(int32_t) * (size_t)p.L * p.E * p.E,
+                            cudaMemcpyDeviceToHost, s);
+    if (e != cudaSuccess) return DO_ERR_CUDA;
+    return do_device_status(ws, stream);
+}
+
+const char *do_status_string(int32_t status) {
+    switch (status) {
+        case DO_OK: return "ok";
+        case DO_ERR_INVALID_ARG: return "invalid argument (null pointer, size or alignment)";
+        case DO_ERR_UNSUPPORTED: return "valid arguments outside this build's limits";
+        case DO_ERR_CUDA: return "a CUDA runtime call or kernel launch failed";
+        case DO_ERR_TIMEOUT: return "a bounded device wait ran out";
+        case DO_ERR_OVERFLOW: return "a row sum of the Hamming matrix does not fit int32";
+        case DO_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+        default: return "unknown status";
+    }
+}
+
+}  // extern "C"

@@ -1,0 +1,215 @@
+"""Python binding of libdoloss (include/doloss.h) over torch CUDA tensors.
+
+Argument marshalling only: every step of the DO-loss path runs in the CUDA
+kernels of libdoloss.so.  torch supplies device memory and the current
+stream.  There is no CPU fallback: if the library is not built, or a call
+fails, these functions raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+GATE_SIGMOID_NORM = 0
+GATE_SOFTMAX = 1
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_build", "libdoloss.so")
+_lock = threading.Lock()
+_lib = None
+
+EXPORTS = {
+    # name: (argtypes, restype)
+    "do_signatures": (["p", "i64", "i32", "i32", "i32", "p", "p", "p"], "i32"),
+    "do_pairwise_hamming": (["p", "i64", "i32", "i32", "p", "p"], "i32"),
+    "do_loss_fwd_bwd": (["p", "p", "p", "i64", "i32", "i32", "i32", "i32", "f32", "f32", "p",
+                         "p", "p", "p", "sz", "p"], "i32"),
+    "do_forward_backward": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p", "p", "p",
+                             "p", "p", "p", "sz", "p"], "i32"),
+    "do_workspace_size": (["i64", "i32", "i32", "i32"], "sz"),
+    "do_device_status": (["p", "p"], "i32"),
+    "do_forward_backward_host": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p", "p",
+                                  "p", "p", "sz", "p"], "i32"),
+    "do_host_buffer_size": (["i64", "i32", "i32", "i32"], "sz"),
+    "do_status_string": (["i32"], "str"),
+}
+
+_CT = {"p": ctypes.c_void_p, "i64": ctypes.c_int64, "i32": ctypes.c_int32,
+       "f32": ctypes.c_float, "sz": ctypes.c_size_t, "str": ctypes.c_char_p}
+
+
+class DoLossError(RuntimeError):
+    def __init__(self, fn: str, status: int):
+        self.status = status
+        super().__init__(f"{fn} failed with status {status}: {status_string(status)}")
+
+
+def lib():
+    """The loaded libdoloss.so; raises if it has not been built."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(LIB_PATH):
+                raise RuntimeError(
+                    f"{LIB_PATH} is missing: build it with "
+                    "`python -c 'import __graft_entry__ as g; g.build()'`")
+            l = ctypes.CDLL(LIB_PATH)
+            for name, (args, res) in EXPORTS.items():
+                fn = getattr(l, name)
+                fn.argtypes = [_CT[a] for a in args]
+                fn.restype = _CT[res]
+            _lib = l
+        return _lib
+
+
+def status_string(status: int) -> str:
+    return lib().do_status_string(int(status)).decode()
+
+
+def _check(fn: str, status: int):
+    if status != 0:
+        raise DoLossError(fn, status)
+
+
+def _stream(t: torch.Tensor) -> int:
+    return torch.cuda.current_stream(t.device).cuda_stream
+
+
+def _ptr(t):
+    return None if t is None else t.data_ptr()
+
+
+def _as3d(logits: torch.Tensor) -> torch.Tensor:
+    if logits.dim() == 2:
+        logits = logits.unsqueeze(0)
+    if logits.dim() != 3 or logits.dtype != torch.float32 or not logits.is_cuda:
+        raise ValueError("logits must be a CUDA float32 tensor of shape [L, T, E] or [T, E]")
+    if not logits.is_contiguous():
+        raise ValueError("logits must be contiguous")
+    return logits
+
+
+def words(T: int) -> int:
+    return (T + 31) // 32
+
+
+def workspace_size(T: int, E: int, k: int, L: int = 1) -> int:
+    return int(lib().do_workspace_size(T, E, k, L))
+
+
+def new_workspace(T: int, E: int, k: int, L: int = 1, device="cuda") -> torch.Tensor:
+    n = workspace_size(T, E, k, L)
+    if n == 0:
+        raise ValueError("invalid sizes")
+    return torch.zeros(n, dtype=torch.uint8, device=device)
+
+
+def signatures(logits: torch.Tensor, k: int, bits=None, counts=None):
+    """Step 1: bits [L,E,W] (int32 storage of uint32 words), counts [L,E] int32."""
+    z = _as3d(logits)
+    L, T, E = z.shape
+    if bits is None:
+        bits = torch.empty(L, E, words(T), dtype=torch.int32, device=z.device)
+    if counts is None:
+        counts = torch.empty(L, E, dtype=torch.int32, device=z.device)
+    _check("do_signatures", lib().do_signatures(z.data_ptr(), T, E, k, L, bits.data_ptr(),
+                                                counts.data_ptr(), _stream(z)))
+    return bits, counts
+
+
+def pairwise_hamming(bits: torch.Tensor, T: int, D=None):
+    """Step 2: D [L,E,E] int32 from bits [L,E,W]."""
+    if bits.dim() == 2:
+        bits = bits.unsqueeze(0)
+    L, E, _ = bits.shape
+    if D is None:
+        D = torch.empty(L, E, E, dtype=torch.int32, device=bits.device)
+    _check("do_pairwise_hamming", lib().do_pairwise_hamming(bits.data_ptr(), T, E, L, D.data_ptr(),
+                                                            _stream(bits)))
+    return D
+
+
+def loss_fwd_bwd(logits, bits, D, k, gate=GATE_SIGMOID_NORM, d_scale=1.0, grad_scale=1.0,
+                 with_grad=True, with_origin=True, workspace=None, dlogits=None):
+    """Step 3: (loss [L] f32, origin_do [L] i64 or None, dlogits [L,T,E] or None)."""
+    z = _as3d(logits)
+    L, T, E = z.shape
+    if bits.dim() == 2:
+        bits = bits.unsqueeze(0)
+    if D.dim() == 2:
+        D = D.unsqueeze(0)
+    loss = torch.empty(L, dtype=torch.float32, device=z.device)
+    origin = torch.empty(L, dtype=torch.int64, device=z.device) if with_origin else None
+    if with_grad and dlogits is None:
+        dlogits = torch.empty_like(z)
+    if not with_grad:
+        dlogits = None
+    if workspace is None:
+        workspace = new_workspace(T, E, k, L, z.device)
+    _check("do_loss_fwd_bwd", lib().do_loss_fwd_bwd(
+        z.data_ptr(), bits.data_ptr(), D.data_ptr(), T, E, k, L, gate, d_scale, grad_scale,
+        loss.data_ptr(), _ptr(origin), _ptr(dlogits), workspace.data_ptr(), workspace.numel(),
+        _stream(z)))
+    return loss, origin, dlogits
+
+
+class Buffers:
+    """Device outputs and workspace of do_forward_backward for one shape."""
+
+    def __init__(self, L, T, E, k, device="cuda", with_grad=True):
+        self.shape = (L, T, E, k)
+        self.bits = torch.empty(L, E, words(T), dtype=torch.int32, device=device)
+        self.counts = torch.empty(L, E, dtype=torch.int32, device=device)
+        self.D = torch.empty(L, E, E, dtype=torch.int32, device=device)
+        self.loss = torch.empty(L, dtype=torch.float32, device=device)
+        self.origin_do = torch.empty(L, dtype=torch.int64, device=device)
+        self.dlogits = torch.empty(L, T, E, dtype=torch.float32, device=device) if with_grad else None
+        self.workspace = new_workspace(T, E, k, L, device)
+
+
+def forward_backward(logits, k, gate=GATE_SIGMOID_NORM, grad_scale=1.0, out: Buffers | None = None,
+                     with_grad=True):
+    """Steps 1-3 in one call; returns the Buffers holding every output."""
+    z = _as3d(logits)
+    L, T, E = z.shape
+    if out is None:
+        out = Buffers(L, T, E, k, z.device, with_grad)
+    if out.shape != (L, T, E, k):
+        raise ValueError("output buffers were made for another shape")
+    dl = out.dlogits if with_grad else None
+    _check("do_forward_backward", lib().do_forward_backward(
+        z.data_ptr(), T, E, k, L, gate, grad_scale, out.bits.data_ptr(), out.counts.data_ptr(),
+        out.D.data_ptr(), out.loss.data_ptr(), out.origin_do.data_ptr(), _ptr(dl),
+        out.workspace.data_ptr(), out.workspace.numel(), _stream(z)))
+    return out
+
+
+def device_status(workspace: torch.Tensor) -> int:
+    """Synchronizes the current stream and returns (and clears) the device status."""
+    return int(lib().do_device_status(workspace.data_ptr(), _stream(workspace)))
+
+
+def host_buffer_size(T, E, k, L=1) -> int:
+    return int(lib().do_host_buffer_size(T, E, k, L))
+
+
+def forward_backward_host(h_logits: torch.Tensor, k, gate=GATE_SIGMOID_NORM, grad_scale=1.0,
+                          device_buffer: torch.Tensor | None = None, h_dlogits=None,
+                          h_counts=None, h_D=None, h_loss=None):
+    """Host arrays in, host arrays out (synchronous), through do_forward_backward_host."""
+    z = h_logits.unsqueeze(0) if h_logits.dim() == 2 else h_logits
+    if z.is_cuda or z.dtype != torch.float32 or not z.is_contiguous():
+        raise ValueError("h_logits must be a contiguous CPU float32 tensor")
+    L, T, E = z.shape
+    if device_buffer is None:
+        device_buffer = torch.empty(host_buffer_size(T, E, k, L), dtype=torch.uint8, device="cuda")
+    if h_loss is None:
+        h_loss = torch.empty(L, dtype=torch.float32)
+    _check("do_forward_backward_host", lib().do_forward_backward_host(
+        z.data_ptr(), T, E, k, L, gate, grad_scale, h_loss.data_ptr(), _ptr(h_dlogits),
+        _ptr(h_counts), _ptr(h_D), device_buffer.data_ptr(), device_buffer.numel(),
+        torch.cuda.current_stream(device_buffer.device).cuda_stream))
+    return h_loss

@@ -1,0 +1,76 @@
+"""The C ABI library loads without a GPU, exports every function that
+include/doloss.h declares, and rejects invalid arguments on the host before
+touching the device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "doloss.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(do_[a-z_0-9]+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def dl():
+    from paper_2609_32398_gb300 import build, doloss
+
+    build.build()
+    return doloss
+
+
+def test_header_declares_the_path(dl):
+    names = declared_functions()
+    for n in ["do_signatures", "do_pairwise_hamming", "do_loss_fwd_bwd", "do_forward_backward"]:
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(dl):
+    lib = ctypes.CDLL(dl.LIB_PATH)
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+        assert name in dl.EXPORTS, f"binding lacks {name}"
+
+
+def test_status_strings(dl):
+    for code in range(7):
+        assert dl.status_string(code)
+    assert dl.status_string(99) == "unknown status"
+
+
+def test_workspace_size_host_logic(dl):
+    assert dl.workspace_size(0, 8, 2, 1) == 0
+    assert dl.workspace_size(10, 8, 9, 1) == 0
+    assert dl.workspace_size(10, 2000, 2, 1) == 0
+    small = dl.workspace_size(1024, 8, 2, 1)
+    big = dl.workspace_size(1 << 20, 256, 8, 48)
+    assert 256 < small < big
+    assert dl.host_buffer_size(1024, 8, 2, 1) > 2 * 4 * 1024 * 8
+
+
+def test_invalid_arguments_are_rejected_before_launch(dl):
+    lib = dl.lib()
+    fake = ctypes.c_void_p(0x10000)           # never dereferenced: validation fails first
+    INV, UNS, WS = 1, 2, 6
+    assert lib.do_signatures(None, 64, 8, 2, 1, fake, fake, None) == INV
+    assert lib.do_signatures(fake, 64, 8, 9, 1, fake, fake, None) == INV     # k > E
+    assert lib.do_signatures(fake, 0, 8, 2, 1, fake, fake, None) == INV      # T = 0
+    assert lib.do_signatures(fake, 64, 2048, 2, 1, fake, fake, None) == UNS  # E > 1024
+    assert lib.do_signatures(fake, 1 << 30, 8, 2, 1, fake, fake, None) == UNS  # (E-1)T >= 2^31
+    odd = ctypes.c_void_p(0x10002)
+    assert lib.do_signatures(odd, 64, 8, 2, 1, fake, fake, None) == INV      # misaligned
+    assert lib.do_pairwise_hamming(fake, 64, 8, 1, None, None) == INV
+    assert lib.do_loss_fwd_bwd(fake, fake, fake, 64, 8, 2, 1, 7, 1.0, 1.0, fake, None, None,
+                               fake, 1 << 20, None) == INV                    # bad gate
+    assert lib.do_loss_fwd_bwd(fake, fake, fake, 64, 8, 2, 1, 0, 1.0, 1.0, fake, None, None,
+                               fake, 8, None) == WS                           # small workspace
+    assert lib.do_forward_backward(fake, 64, 8, 2, 1, 0, 1.0, fake, fake, fake, fake, None, None,
+                                   None, 0, None) == WS
+    assert lib.do_forward_backward_host(None, 64, 8, 2, 1, 0, 1.0, fake, None, None, None, fake,
+                                        1 << 30, None) == INV

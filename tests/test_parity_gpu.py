@@ -1,0 +1,176 @@
+"""Parity of the CUDA path (through the C ABI) with the CPU oracle.
+
+Bits, counts, the Hamming matrix and origin_do must be bit-exact; the loss
+within 1e-5 relative; dlogits within 1e-4 of the oracle's largest entry
+(max-abs normalised).  Inputs are the seeded workloads, drawn once and given
+byte for byte to both sides.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_32398_gb300 import workloads
+
+pytestmark = pytest.mark.gpu
+
+LOSS_RTOL = 1e-5
+GRAD_TOL = 1e-4
+U32 = 2.0 ** -24   # fp32 unit roundoff
+
+
+def loss_tolerance(ref_loss, z, f, D, k, gate, d_scale=1.0):
+    """1e-5 relative, floored by the fp32 accumulation bound of the kernel:
+    each token's sum_i p_it w_it is summed in fp32 over E terms, so its error is
+    below E u sum_i |p_it w_it|; over all tokens that is E u M with
+    M = sum_t sum_i p_it |dL/dp_it| (exact zeros such as uniform p need it)."""
+    T, E = z.shape
+    M = float((oracle.gate(z, gate) * np.abs(oracle.dloss_dp(D, f, T, k, d_scale))).sum())
+    return max(LOSS_RTOL * abs(ref_loss), E * U32 * M)
+
+
+@pytest.fixture(scope="module")
+def dl():
+    import paper_2609_32398_gb300.doloss as m
+
+    m.lib()
+    return m
+
+
+def gpu_run(dl, z_cpu, k, gate, grad_scale=1.0):
+    z = z_cpu.to("cuda")
+    out = dl.forward_backward(z, k, gate=gate, grad_scale=grad_scale)
+    st = dl.device_status(out.workspace)
+    assert st == 0, dl.status_string(st)
+    return out
+
+
+def assert_layer(out, l, zl, k, gate, grad_scale=1.0):
+    ref = oracle.forward_backward(zl, k, gate, grad_scale=grad_scale)
+    bits = out.bits[l].cpu().numpy().view(np.uint32)
+    assert np.array_equal(bits, ref["bits"]), "signatures"
+    assert np.array_equal(out.counts[l].cpu().numpy(), ref["counts"]), "counts"
+    assert np.array_equal(out.D[l].cpu().numpy(), ref["D"]), "Hamming matrix"
+    assert int(out.origin_do[l]) == ref["origin_do"], "origin_do"
+    loss = float(out.loss[l])
+    tol = LOSS_RTOL * abs(ref["loss"])
+    if abs(loss - ref["loss"]) > tol:
+        tol = loss_tolerance(ref["loss"], zl, oracle.select(zl, k), ref["D"], k, gate)
+    assert abs(loss - ref["loss"]) <= tol, ("loss", loss, ref["loss"], tol)
+    g = out.dlogits[l].double().cpu().numpy()
+    scale = np.abs(ref["dz"]).max()
+    err = np.abs(g - ref["dz"]).max() / scale if scale > 0 else np.abs(g).max()
+    assert err <= GRAD_TOL, f"dlogits error {err:.3e}"
+
+
+@pytest.mark.parametrize("gate", [workloads.GATE_SOFTMAX, workloads.GATE_SIGMOID_NORM])
+def test_tiny_full_size(dl, gate):
+    w = workloads.get("tiny")
+    z = workloads.logits(w)
+    out = gpu_run(dl, z, w.k, gate)
+    assert_layer(out, 0, z[0].numpy(), w.k, gate)
+
+
+@pytest.mark.parametrize("name,T,L", [("c2", None, None), ("c3", 8192 + 19, None),
+                                      ("collapse", 16384 + 5, None), ("long", 4096 + 7, 3)])
+def test_workload_recipes_reduced(dl, name, T, L):
+    w = workloads.get(name, T=T, L=L)
+    z = workloads.logits(w)
+    out = gpu_run(dl, z, w.k, w.gate, grad_scale=1e-5 if name == "c3" else 1.0)
+    for l in range(w.L):
+        assert_layer(out, l, z[l].numpy(), w.k, w.gate, grad_scale=1e-5 if name == "c3" else 1.0)
+
+
+def test_c3_full_size_elementwise(dl):
+    """E=128, k=8, T=65536 -- the benchmark workload -- element by element."""
+    w = workloads.get("c3")
+    z = workloads.logits(w)
+    out = gpu_run(dl, z, w.k, w.gate)
+    assert_layer(out, 0, z[0].numpy(), w.k, w.gate)
+
+
+@pytest.mark.parametrize(
+    "T,E,k,L,gate,ties",
+    [(1, 1, 1, 1, 0, False), (1, 5, 3, 2, 1, False), (31, 8, 8, 1, 0, True), (33, 33, 1, 1, 0, True),
+     (100, 100, 7, 2, 1, True), (777, 64, 64, 1, 0, False), (1000, 200, 16, 1, 0, True),
+     (513, 256, 8, 2, 0, True), (300, 1024, 8, 1, 0, False), (64, 37, 36, 1, 1, True),
+     (2049, 96, 5, 1, 0, False)])
+def test_edge_shapes(dl, T, E, k, L, gate, ties):
+    z = workloads.random_logits(T, E, L=L, seed=T * 7 + E, ties=ties)
+    out = gpu_run(dl, z, k, gate, grad_scale=0.5)
+    for l in range(L):
+        assert_layer(out, l, z[l].numpy(), k, gate, grad_scale=0.5)
+
+
+def test_all_equal_logits_select_lowest_indices(dl):
+    T, E, k = 96, 40, 6
+    z = torch.full((1, T, E), 0.75)
+    out = gpu_run(dl, z, k, 0)
+    f = np.zeros((T, E), np.uint8)
+    f[:, :k] = 1
+    assert np.array_equal(out.bits[0].cpu().numpy().view(np.uint32), oracle.pack(f))
+    assert float(out.loss[0]) == pytest.approx(0.0, abs=1e-7)    # p uniform -> L = 0
+    assert_layer(out, 0, z[0].numpy(), k, 0)
+
+
+def test_split_api_matches_fused_and_is_deterministic(dl):
+    w = workloads.get("c2", T=5000)
+    z = workloads.logits(w).cuda()
+    fused = dl.forward_backward(z, w.k, w.gate)
+    bits, counts = dl.signatures(z, w.k)
+    D = dl.pairwise_hamming(bits, w.T)
+    loss, origin, dz = dl.loss_fwd_bwd(z, bits, D, w.k, w.gate)
+    again = dl.forward_backward(z, w.k, w.gate)
+    torch.cuda.synchronize()
+    for a, b in [(fused.bits, bits), (fused.counts, counts), (fused.D, D), (fused.loss, loss),
+                 (fused.origin_do, origin), (fused.dlogits, dz), (fused.dlogits, again.dlogits),
+                 (fused.loss, again.loss)]:
+        assert torch.equal(a, b)
+
+
+def test_global_do_summed_matrix_with_d_scale(dl):
+    """Eq. global_do: two replicas' Hamming matrices summed, scaled by 1/2, applied
+    to one replica's local direction term."""
+    T, E, k = 3000, 64, 4
+    z = workloads.random_logits(2 * T, E, seed=99).reshape(2, T, E)
+    zc = z.cuda()
+    b0, _ = dl.signatures(zc[0], k)
+    b1, _ = dl.signatures(zc[1], k)
+    Dsum = dl.pairwise_hamming(b0, T) + dl.pairwise_hamming(b1, T)
+    loss, _, dz = dl.loss_fwd_bwd(zc[0], b0, Dsum, k, 0, d_scale=0.5, grad_scale=2.0)
+    torch.cuda.synchronize()
+    z0 = z[0].numpy()
+    f0 = oracle.select(z0, k)
+    D = oracle.hamming(f0) + oracle.hamming(oracle.select(z[1].numpy(), k))
+    assert np.array_equal(Dsum[0].cpu().numpy(), D)
+    ref = oracle.loss(D, oracle.direction(z0, f0), T, k, d_scale=0.5)
+    assert float(loss[0]) == pytest.approx(ref, rel=LOSS_RTOL)
+    rdz = oracle.gate_backward(z0, oracle.dloss_dp(D, f0, T, k, d_scale=0.5), grad_scale=2.0)
+    err = np.abs(dz[0].double().cpu().numpy() - rdz).max() / np.abs(rdz).max()
+    assert err <= GRAD_TOL
+
+
+def test_row_sum_overflow_is_reported(dl):
+    T, E, k = 64, 8, 2
+    z = workloads.random_logits(T, E, seed=5).cuda()
+    bits, _ = dl.signatures(z, k)
+    D = torch.full((1, E, E), 1 << 29, dtype=torch.int32, device="cuda")
+    ws = dl.new_workspace(T, E, k)
+    dl.loss_fwd_bwd(z, bits, D, k, 0, workspace=ws)
+    assert dl.device_status(ws) == 5          # DO_ERR_OVERFLOW
+    assert dl.device_status(ws) == 0          # cleared after reading
+
+
+def test_host_entry_point_matches_device_path(dl):
+    w = workloads.get("c2", T=4000)
+    z = workloads.logits(w)
+    hz = z.pin_memory()
+    h_dz = torch.empty_like(hz).pin_memory()
+    h_counts = torch.empty(1, w.E, dtype=torch.int32)
+    h_D = torch.empty(1, w.E, w.E, dtype=torch.int32)
+    h_loss = dl.forward_backward_host(hz, w.k, w.gate, h_dlogits=h_dz, h_counts=h_counts, h_D=h_D)
+    dev = gpu_run(dl, z, w.k, w.gate)
+    assert torch.equal(h_loss, dev.loss.cpu())
+    assert torch.equal(h_dz, dev.dlogits.cpu())
+    assert torch.equal(h_counts, dev.counts.cpu())
+    assert torch.equal(h_D, dev.D.cpu())
