@@ -61,7 +61,15 @@ do_status do_signatures(const float *logits, int64_t T, int32_t E, int32_t k, in
     if (st != DO_OK) return st;
     if (!logits || !bits || !counts) return DO_ERR_INVALID_ARG;
     if (!aligned(logits, 4) || !aligned(bits, 4) || !aligned(counts, 4)) return DO_ERR_INVALID_ARG;
-    return from_cuda(dol::launch_signatures(logits, p, bits, counts, (cudaStream_t)stream));
+    cudaStream_t s = (cudaStream_t)stream;
+    if (dol::signatures_fast_supported(logits, p)) {
+        cudaError_t e = cudaMemsetAsync(counts, 0, sizeof(int) * (size_t)p.L * p.E, s);
+        const dol::ZeroSpans none = {{nullptr, nullptr, nullptr}, {0, 0, 0}};
+        if (e == cudaSuccess)
+            e = dol::launch_signatures_fast(logits, p, bits, counts, nullptr, none, nullptr, s);
+        return from_cuda(e);
+    }
+    return from_cuda(dol::launch_signatures(logits, p, bits, counts, s));
 }
 
 do_status do_pairwise_hamming(const uint32_t *bits, int64_t T, int32_t E, int32_t L, int32_t *D,
@@ -89,9 +97,23 @@ do_status do_loss_fwd_bwd(const float *logits, const uint32_t *bits, const int32
         return DO_ERR_INVALID_ARG;
     if (!workspace || !aligned(workspace, 256) || workspace_bytes < dol::workspace_bytes(p))
         return DO_ERR_WORKSPACE;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (dol::loss_fast_supported(p, logits, D, dlogits) && aligned(bits, 16)) {
+        const dol::WsLayout w = dol::ws_layout(p);
+        char *ws = static_cast<char *>(workspace);
+        int *done = reinterpret_cast<int *>(ws + w.done);
+        uint8_t *idx = reinterpret_cast<uint8_t *>(ws + w.idx);
+        cudaError_t e = dol::launch_idx_from_bits(bits, p, idx, done, p.L, s);
+        if (e == cudaSuccess)
+            e = dol::launch_loss_fast(logits, idx, D, p, gate, d_scale, grad_scale, loss,
+                                      reinterpret_cast<long long *>(origin_do), dlogits,
+                                      reinterpret_cast<double *>(ws + w.partials), done,
+                                      reinterpret_cast<int *>(ws), s);
+        return from_cuda(e);
+    }
     return from_cuda(dol::launch_loss(logits, bits, D, p, gate, d_scale, grad_scale, loss,
                                       reinterpret_cast<long long *>(origin_do), dlogits,
-                                      workspace, (cudaStream_t)stream));
+                                      workspace, s));
 }
 
 do_status do_forward_backward(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
@@ -111,6 +133,24 @@ do_status do_forward_backward(const float *logits, int64_t T, int32_t E, int32_t
     if (!workspace || !aligned(workspace, 256) || workspace_bytes < dol::workspace_bytes(p))
         return DO_ERR_WORKSPACE;
     cudaStream_t s = (cudaStream_t)stream;
+    if (dol::signatures_fast_supported(logits, p) && dol::loss_fast_supported(p, logits, D, dlogits) &&
+        aligned(bits, 16)) {
+        // signatures (which clear D, counts and the done counters) -> Hamming -> loss
+        const dol::WsLayout w = dol::ws_layout(p);
+        char *ws = static_cast<char *>(workspace);
+        int *done = reinterpret_cast<int *>(ws + w.done);
+        uint8_t *idx = reinterpret_cast<uint8_t *>(ws + w.idx);
+        const dol::ZeroSpans zero = {{D, counts, done},
+                                     {(int64_t)p.L * p.E * p.E, (int64_t)p.L * p.E, (int64_t)p.L}};
+        int *status = reinterpret_cast<int *>(ws);
+        cudaError_t e = dol::launch_signatures_fast(logits, p, bits, nullptr, idx, zero, status, s);
+        if (e == cudaSuccess) e = dol::launch_hamming_accumulate(bits, p, D, counts, s);
+        if (e == cudaSuccess)
+            e = dol::launch_loss_fast(logits, idx, D, p, gate, 1.0f, grad_scale, loss,
+                                      reinterpret_cast<long long *>(origin_do), dlogits,
+                                      reinterpret_cast<double *>(ws + w.partials), done, status, s);
+        return from_cuda(e);
+    }
     cudaError_t e = dol::launch_signatures(logits, p, bits, counts, s);
     if (e == cudaSuccess) e = dol::launch_hamming(bits, p, D, s);
     if (e == cudaSuccess)

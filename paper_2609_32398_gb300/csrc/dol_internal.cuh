@@ -26,19 +26,51 @@ struct Problem {
     int64_t W;    // 32-bit words per signature, ceil(T/32)
 };
 
-// Number of loss-kernel CTAs per problem; fixes the partial-sum layout and
-// therefore the reduction order (deterministic for given T, E, L).
+// Up to three int ranges that a kernel clears for the kernels after it.
+struct ZeroSpans {
+    int *p[3];
+    int64_t n[3];
+};
+
+// Workspace of the loss step, carved from the caller's buffer:
+//   [0, 256)        device status word (kDevOverflow | kDevTimeout bits)
+//   done            [L] int, per-problem count of finished loss CTAs
+//   partials        [L][max CTAs per problem] fp64 sums of A_t
+//   idx             [L][T][k] uint8, the selected experts of every token
+struct WsLayout {
+    size_t done, partials, idx, total;
+    int max_parts;  // partial slots per problem
+};
+WsLayout ws_layout(const Problem &p);
+inline size_t workspace_bytes(const Problem &p) { return ws_layout(p).total; }
+
+// Number of generic loss-kernel CTAs per problem; fixes the partial-sum
+// layout and therefore the reduction order.
 int loss_blocks_per_problem(const Problem &p);
-size_t workspace_bytes(const Problem &p);
 
 // Launchers (return the first CUDA error, cudaSuccess otherwise).
 cudaError_t launch_signatures(const float *logits, const Problem &p, uint32_t *bits,
                               int *counts, cudaStream_t s);
 cudaError_t launch_hamming(const uint32_t *bits, const Problem &p, int *D, cudaStream_t s);
+cudaError_t launch_hamming_accumulate(const uint32_t *bits, const Problem &p, int *D, int *counts,
+                                      cudaStream_t s);
 cudaError_t launch_loss(const float *logits, const uint32_t *bits, const int *D,
                         const Problem &p, int gate, float d_scale, float grad_scale,
                         float *loss, long long *origin_do, float *dlogits, void *workspace,
                         cudaStream_t s);
+
+// Fast paths (E in {32, 64, 128}, k in {1, 2, 4, 8}, 16-byte aligned rows).
+bool signatures_fast_supported(const float *logits, const Problem &p);
+cudaError_t launch_signatures_fast(const float *logits, const Problem &p, uint32_t *bits,
+                                   int *counts, uint8_t *idx, const ZeroSpans &zero, int *status,
+                                   cudaStream_t s);
+bool loss_fast_supported(const Problem &p, const float *logits, const int *D, const float *dlogits);
+cudaError_t launch_idx_from_bits(const uint32_t *bits, const Problem &p, uint8_t *idx, int *zero_ptr,
+                                 int zero_n, cudaStream_t s);
+cudaError_t launch_loss_fast(const float *logits, const uint8_t *idx, const int *D, const Problem &p,
+                             int gate, float d_scale, float grad_scale, float *loss,
+                             long long *origin_do, float *dlogits, double *partials, int *done,
+                             int *status, cudaStream_t s);
 
 // ---------------------------------------------------------------- device helpers
 

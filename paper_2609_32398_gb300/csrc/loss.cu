@@ -230,15 +230,26 @@ int loss_blocks_per_problem(const Problem &p) {
     return (int)(blocks < 1 ? 1 : blocks);
 }
 
-size_t workspace_bytes(const Problem &p) {
-    return kWsHeader + sizeof(double) * (size_t)p.L * (size_t)loss_blocks_per_problem(p);
+WsLayout ws_layout(const Problem &p) {
+    auto up = [](size_t x) { return (x + 255) / 256 * 256; };
+    WsLayout w;
+    const int64_t fast_parts = p.W;  // the fast kernel gives every CTA at least 32 tokens
+    const int64_t gen_parts = loss_blocks_per_problem(p);
+    w.max_parts = (int)(fast_parts > gen_parts ? fast_parts : gen_parts);
+    const bool fast_k = p.k == 1 || p.k == 2 || p.k == 4 || p.k == 8;
+    w.done = kWsHeader;
+    w.partials = up(w.done + sizeof(int) * (size_t)p.L);
+    w.idx = up(w.partials + sizeof(double) * (size_t)p.L * (size_t)w.max_parts);
+    w.total = up(w.idx + (fast_k ? (size_t)p.L * (size_t)p.T * (size_t)p.k : 0));
+    return w;
 }
 
 cudaError_t launch_loss(const float *logits, const uint32_t *bits, const int *D, const Problem &p,
                         int gate, float d_scale, float grad_scale, float *loss,
                         long long *origin_do, float *dlogits, void *workspace, cudaStream_t s) {
     int *status = reinterpret_cast<int *>(workspace);
-    double *partials = reinterpret_cast<double *>(static_cast<char *>(workspace) + kWsHeader);
+    double *partials =
+        reinterpret_cast<double *>(static_cast<char *>(workspace) + ws_layout(p).partials);
     const int P = loss_blocks_per_problem(p);
     const double norm = 1.0 / ((double)p.T * (double)p.T * (double)p.k);
     const float coef = (float)((double)grad_scale * (double)d_scale * norm);

@@ -1,0 +1,406 @@
+// Step 3, fast path (E in {32, 64, 128}, k in {1, 2, 4, 8}): the surrogate
+// DO-loss and its gradient (Sec. 3.1.3, Eq. do_loss; Eq. global_do scaling).
+//
+// With R_i = sum_j D_ij, put D'_ij = D_ij off the diagonal and D'_ii = -R_i.
+// Then for the k experts S_t of token t
+//   sum_{j in S_t} D'_ji = sum_{j in S_t} D_ji - f_it R_i = -w_it,
+// the integer weight w_it = sum_j D_ij (f_it - f_jt) whose product with
+// d_scale/(m^2 k) is dL/dp_it.  One k-row gather of D' per token therefore
+// gives every w_it without looking at the signature bits.  D must be
+// symmetric (every Hamming matrix and every sum of them is).
+//
+// Layout: a CTA copies D into shared memory once (bulk copy), writes the
+// diagonal -R_i, then its warps walk tokens with G = E/16 lanes per token;
+// lane g of a token group owns experts c*E/4 + 4g .. +3 for c = 0..3, so the
+// group reads 16-byte chunks of the logits row, of the D' rows and writes the
+// dlogits row with coalesced 16-byte accesses.  Per token:
+//   sigmoid-norm  s = sigmoid(z), A = sum s w / sum s,
+//                 dz = c s (1 - s) (w - A) / sum s
+//   softmax       e = exp(z - max), A = sum e w / sum e, dz = c e (w - A) / sum e
+// with c = grad_scale d_scale / (m^2 k).  A is summed per CTA in fp64 and the
+// last CTA of each problem adds the CTA partials in index order.
+#include <climits>
+
+#include "dol_internal.cuh"
+#include "tma.cuh"
+
+namespace dol {
+namespace {
+
+constexpr int kLossFastThreads = 256;
+constexpr int kLossFastWarps = kLossFastThreads / 32;
+
+__device__ __forceinline__ float sigmoid_fast(float z) {
+    const float e = __expf(-fmaxf(z, -80.0f));
+    return __fdividef(1.0f, 1.0f + e);
+}
+
+template <int K>
+__device__ __forceinline__ void load_idx(const uint8_t *p, int (&j)[K]) {
+    if (K == 8) {
+        const uint2 v = __ldg(reinterpret_cast<const uint2 *>(p));
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            j[q % K] = (v.x >> (8 * q)) & 0xff;
+            j[(4 + q) % K] = (v.y >> (8 * q)) & 0xff;
+        }
+    } else if (K == 4) {
+        const uint32_t v = __ldg(reinterpret_cast<const uint32_t *>(p));
+#pragma unroll
+        for (int q = 0; q < K; ++q) j[q] = (v >> (8 * q)) & 0xff;
+    } else if (K == 2) {
+        const uint32_t v = __ldg(reinterpret_cast<const uint16_t *>(p));
+        j[0] = v & 0xff;
+        j[1 % K] = (v >> 8) & 0xff;
+    } else {
+        j[0] = __ldg(p);
+    }
+}
+
+template <int E, int K, int kGate>
+__global__ void __launch_bounds__(kLossFastThreads)
+loss_fast_kernel(const float *__restrict__ logits, const uint8_t *__restrict__ idx,
+                 const int *__restrict__ Dg, int64_t T, int tokens_per_cta, float coef,
+                 double scale, float *__restrict__ dlogits, double *__restrict__ partials,
+                 int *__restrict__ done, float *__restrict__ loss, long long *__restrict__ origin_do,
+                 int *__restrict__ status) {
+    constexpr int G = E / 16;       // lanes per token
+    constexpr int TPW = 32 / G;     // tokens per warp pass
+    constexpr int Q = E / 4;        // expert stride between a lane's chunks
+    extern __shared__ __align__(128) int sD[];  // [E][E]
+    __shared__ __align__(8) uint64_t bar;
+    __shared__ double s_part[kLossFastWarps];
+    __shared__ int s_last;
+
+    const int layer = blockIdx.y;
+    const int P = gridDim.x;
+    const int *Dl = Dg + (int64_t)layer * E * E;
+
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        fence_barrier_init();
+    }
+    __syncthreads();
+    pdl_wait();  // D, idx and the zeroed counters come from the previous kernels
+    if (threadIdx.x == 0) {
+        mbar_arrive_expect_tx(&bar, (uint32_t)(sizeof(int) * E * E));
+        bulk_load(sD, Dl, (uint32_t)(sizeof(int) * E * E), &bar);
+    }
+    const bool have_d = mbar_wait(&bar, 0, status);
+    if (__syncthreads_or(!have_d)) return;
+    if (threadIdx.x < E) {
+        const int i = threadIdx.x;
+        long long r = 0;
+        for (int j = 0; j < E; ++j) r += sD[j * E + i];
+        if (r > INT_MAX || r < 0) atomicOr(status, kDevOverflow);
+        sD[i * E + i] = -(int)r;
+    }
+    __syncthreads();
+
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int grp = lane / G, g = lane % G;
+    const float *zl = logits + (int64_t)layer * T * E;
+    float *dzl = dlogits ? dlogits + (int64_t)layer * T * E : nullptr;
+    const uint8_t *il = idx + (int64_t)layer * T * K;
+    const int64_t t_begin = (int64_t)blockIdx.x * tokens_per_cta;
+    const int64_t t_end = min64(T, t_begin + tokens_per_cta);
+    double tok_sum = 0.0;
+
+    for (int64_t tb = t_begin + (int64_t)warp * TPW; tb < t_end; tb += (int64_t)kLossFastWarps * TPW) {
+        const int64_t t = tb + grp;
+        const bool valid = t < t_end;
+        const int64_t tc = valid ? t : t_begin;  // clamp: invalid lanes recompute a valid token
+        int js[K];
+        load_idx<K>(il + tc * K, js);
+        float4 zc[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+            zc[c] = __ldg(reinterpret_cast<const float4 *>(zl + tc * E + c * Q + 4 * g));
+        int4 acc[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[c] = make_int4(0, 0, 0, 0);
+#pragma unroll
+        for (int q = 0; q < K; ++q) {
+            const int *row = sD + js[q] * E + 4 * g;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                const int4 d = *reinterpret_cast<const int4 *>(row + c * Q);
+                acc[c].x += d.x;
+                acc[c].y += d.y;
+                acc[c].z += d.z;
+                acc[c].w += d.w;
+            }
+        }
+        float w[16], zz[16], gv[16];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            w[4 * c] = -(float)acc[c].x;
+            w[4 * c + 1] = -(float)acc[c].y;
+            w[4 * c + 2] = -(float)acc[c].z;
+            w[4 * c + 3] = -(float)acc[c].w;
+            zz[4 * c] = zc[c].x;
+            zz[4 * c + 1] = zc[c].y;
+            zz[4 * c + 2] = zc[c].z;
+            zz[4 * c + 3] = zc[c].w;
+        }
+        float den = 0.0f, num = 0.0f;
+        if (kGate == 0) {
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                gv[e] = sigmoid_fast(zz[e]);
+                den += gv[e];
+                num = fmaf(gv[e], w[e], num);
+            }
+        } else {
+            float mx = zz[0];
+#pragma unroll
+            for (int e = 1; e < 16; ++e) mx = fmaxf(mx, zz[e]);
+#pragma unroll
+            for (int o = G / 2; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, o));
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                gv[e] = __expf(zz[e] - mx);
+                den += gv[e];
+                num = fmaf(gv[e], w[e], num);
+            }
+        }
+#pragma unroll
+        for (int o = G / 2; o > 0; o >>= 1) {
+            den += __shfl_xor_sync(kFull, den, o);
+            num += __shfl_xor_sync(kFull, num, o);
+        }
+        const float inv = 1.0f / den;
+        const float A = num * inv;
+        if (valid && g == 0) tok_sum += (double)A;
+        if (dzl && valid) {
+            const float cs = coef * inv;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                float4 o;
+                float *op = reinterpret_cast<float *>(&o);
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float s = gv[4 * c + e];
+                    const float jac = (kGate == 0) ? s - s * s : s;
+                    op[e] = cs * jac * (w[4 * c + e] - A);
+                }
+                *reinterpret_cast<float4 *>(dzl + t * E + c * Q + 4 * g) = o;
+            }
+        }
+    }
+    // CTA partial, in warp and lane order
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) tok_sum += __shfl_xor_sync(kFull, tok_sum, o);
+    if (lane == 0) s_part[warp] = tok_sum;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double sum = 0.0;
+        for (int q = 0; q < kLossFastWarps; ++q) sum += s_part[q];
+        partials[(int64_t)layer * P + blockIdx.x] = sum;
+        __threadfence();
+        s_last = (atomicAdd(&done[layer], 1) == P - 1);
+    }
+    __syncthreads();
+    if (!s_last) return;
+    // last CTA of this problem: fixed-order sum of the partials, origin_do
+    __threadfence();
+    if (threadIdx.x == 0) {
+        const volatile double *pp = partials + (int64_t)layer * P;
+        double sum = 0.0;
+        for (int b = 0; b < P; ++b) sum += pp[b];
+        loss[layer] = (float)(sum * scale);
+        done[layer] = 0;
+    }
+    if (origin_do) {
+        long long o = 0;
+        for (int e = threadIdx.x; e < E * E; e += blockDim.x) {
+            const int i = e / E, j = e - (e / E) * E;
+            if (i != j) {
+                const long long d = sD[e];
+                o += d * d;
+            }
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) o += __shfl_xor_sync(kFull, o, off);
+        __shared__ long long s_o[kLossFastWarps];
+        if (lane == 0) s_o[warp] = o;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            long long sum = 0;
+            for (int q = 0; q < kLossFastWarps; ++q) sum += s_o[q];
+            origin_do[layer] = sum;
+        }
+    }
+}
+
+// Selected-expert indices of every token recovered from the signature words
+// (for do_loss_fwd_bwd, whose caller passes bits): a warp per 32-token tile
+// transposes the E/32 words back to one row per token and lists its set bits.
+template <int E, int K>
+__global__ void __launch_bounds__(256)
+idx_from_bits_kernel(const uint32_t *__restrict__ bits, int64_t T, int64_t W, int64_t ntiles,
+                     uint8_t *__restrict__ idx, int *__restrict__ zero_ptr, int zero_n) {
+    constexpr int R = E / 32;
+    pdl_trigger();
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < zero_n; i += gridDim.x * blockDim.x)
+        zero_ptr[i] = 0;
+    const int lane = threadIdx.x & 31;
+    const int64_t wid = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const uint32_t lo_mask[5] = {0x0000FFFFu, 0x00FF00FFu, 0x0F0F0F0Fu, 0x33333333u, 0x55555555u};
+    for (int64_t tile = wid; tile < ntiles; tile += nw) {
+        const int64_t layer = tile / W, w = tile - layer * W;
+        uint32_t m[R];
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            uint32_t x = __ldg(bits + (layer * E + 32 * r + lane) * W + w);
+            // lane = expert column -> lane = token row (the same bit transpose)
+#pragma unroll
+            for (int s = 0; s < 5; ++s) {
+                const int j = 16 >> s;
+                const uint32_t lo = lo_mask[s];
+                const uint32_t p = __shfl_xor_sync(kFull, x, j);
+                x = (lane & j) ? ((x & ~lo) | ((p >> j) & lo)) : ((x & lo) | ((p << j) & ~lo));
+            }
+            m[r] = x;
+        }
+        const int64_t t = 32 * w + lane;
+        if (t >= T) continue;
+        uint8_t out[K];
+        int n = 0;
+#pragma unroll
+        for (int q = 0; q < K; ++q) out[q] = 0;
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            uint32_t x = m[r];
+            while (x && n < K) {
+                const int b = __ffs(x) - 1;
+                x &= x - 1;
+#pragma unroll
+                for (int q = 0; q < K; ++q)
+                    if (q == n) out[q] = (uint8_t)(32 * r + b);
+                ++n;
+            }
+        }
+        uint8_t *p = idx + (layer * T + t) * K;
+#pragma unroll
+        for (int q = 0; q < K; ++q) p[q] = out[q];
+    }
+}
+
+template <int E, int K>
+cudaError_t run_loss_fast(const float *logits, const uint8_t *idx, const int *D, const Problem &p,
+                          int gate, float coef, double scale, float *dlogits, double *partials,
+                          int P, int tokens_per_cta, int *done, float *loss, long long *origin_do,
+                          int *status, cudaStream_t s) {
+    const size_t smem = sizeof(int) * E * E;
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(loss_fast_kernel<E, K, 0>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(loss_fast_kernel<E, K, 1>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)P, (unsigned)p.L);
+    cfg.blockDim = dim3(kLossFastThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (gate == 0)
+        return cudaLaunchKernelEx(&cfg, loss_fast_kernel<E, K, 0>, logits, idx, D, p.T, tokens_per_cta,
+                                  coef, scale, dlogits, partials, done, loss, origin_do, status);
+    return cudaLaunchKernelEx(&cfg, loss_fast_kernel<E, K, 1>, logits, idx, D, p.T, tokens_per_cta,
+                              coef, scale, dlogits, partials, done, loss, origin_do, status);
+}
+
+template <int E>
+cudaError_t dispatch_loss_k(const float *logits, const uint8_t *idx, const int *D, const Problem &p,
+                            int gate, float coef, double scale, float *dlogits, double *partials,
+                            int P, int tpc, int *done, float *loss, long long *origin_do, int *status,
+                            cudaStream_t s) {
+    switch (p.k) {
+        case 1: return run_loss_fast<E, 1>(logits, idx, D, p, gate, coef, scale, dlogits, partials, P, tpc, done, loss, origin_do, status, s);
+        case 2: return run_loss_fast<E, 2>(logits, idx, D, p, gate, coef, scale, dlogits, partials, P, tpc, done, loss, origin_do, status, s);
+        case 4: return run_loss_fast<E, 4>(logits, idx, D, p, gate, coef, scale, dlogits, partials, P, tpc, done, loss, origin_do, status, s);
+        default: return run_loss_fast<E, 8>(logits, idx, D, p, gate, coef, scale, dlogits, partials, P, tpc, done, loss, origin_do, status, s);
+    }
+}
+
+template <int E, int K>
+cudaError_t run_idx(const uint32_t *bits, const Problem &p, uint8_t *idx, int *zero_ptr, int zero_n,
+                    cudaStream_t s) {
+    const int64_t ntiles = (int64_t)p.L * p.W;
+    int64_t blocks = (ntiles + 7) / 8;
+    if (blocks > 4096) blocks = 4096;
+    idx_from_bits_kernel<E, K><<<(unsigned)blocks, 256, 0, s>>>(bits, p.T, p.W, ntiles, idx, zero_ptr,
+                                                                zero_n);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+bool loss_fast_supported(const Problem &p, const float *logits, const int *D, const float *dlogits) {
+    const bool e_ok = p.E == 32 || p.E == 64 || p.E == 128;
+    const bool k_ok = p.k == 1 || p.k == 2 || p.k == 4 || p.k == 8;
+    return e_ok && k_ok && reinterpret_cast<uintptr_t>(logits) % 16 == 0 &&
+           reinterpret_cast<uintptr_t>(D) % 16 == 0 &&
+           (dlogits == nullptr || reinterpret_cast<uintptr_t>(dlogits) % 16 == 0);
+}
+
+// CTAs per problem of the fast loss kernel and the tokens each one takes.
+void loss_fast_grid(const Problem &p, int *P, int *tokens_per_cta) {
+    int dev = 0, sms = 148;
+    if (cudaGetDevice(&dev) == cudaSuccess)
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    int64_t want = (int64_t)sms * 3 / p.L;
+    if (want < 1) want = 1;
+    int64_t tpc = (p.T + want - 1) / want;
+    tpc = (tpc + 31) / 32 * 32;
+    if (tpc < 32) tpc = 32;
+    *tokens_per_cta = (int)tpc;
+    *P = (int)((p.T + tpc - 1) / tpc);
+}
+
+cudaError_t launch_idx_from_bits(const uint32_t *bits, const Problem &p, uint8_t *idx, int *zero_ptr,
+                                 int zero_n, cudaStream_t s) {
+#define DOL_IDX_CASE(EE)                                                          \
+    if (p.E == EE) {                                                              \
+        switch (p.k) {                                                            \
+            case 1: return run_idx<EE, 1>(bits, p, idx, zero_ptr, zero_n, s);     \
+            case 2: return run_idx<EE, 2>(bits, p, idx, zero_ptr, zero_n, s);     \
+            case 4: return run_idx<EE, 4>(bits, p, idx, zero_ptr, zero_n, s);     \
+            default: return run_idx<EE, 8>(bits, p, idx, zero_ptr, zero_n, s);    \
+        }                                                                         \
+    }
+    DOL_IDX_CASE(32)
+    DOL_IDX_CASE(64)
+    DOL_IDX_CASE(128)
+#undef DOL_IDX_CASE
+    return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_loss_fast(const float *logits, const uint8_t *idx, const int *D, const Problem &p,
+                             int gate, float d_scale, float grad_scale, float *loss,
+                             long long *origin_do, float *dlogits, double *partials, int *done,
+                             int *status, cudaStream_t s) {
+    int P = 1, tpc = 32;
+    loss_fast_grid(p, &P, &tpc);
+    const double norm = 1.0 / ((double)p.T * (double)p.T * (double)p.k);
+    const float coef = (float)((double)grad_scale * (double)d_scale * norm);
+    const double scale = (double)d_scale * norm;
+    if (p.E == 32)
+        return dispatch_loss_k<32>(logits, idx, D, p, gate, coef, scale, dlogits, partials, P, tpc, done, loss, origin_do, status, s);
+    if (p.E == 64)
+        return dispatch_loss_k<64>(logits, idx, D, p, gate, coef, scale, dlogits, partials, P, tpc, done, loss, origin_do, status, s);
+    return dispatch_loss_k<128>(logits, idx, D, p, gate, coef, scale, dlogits, partials, P, tpc, done, loss, origin_do, status, s);
+}
+
+}  // namespace dol

@@ -1,0 +1,347 @@
+// Step 1, fast path (E in {32, 64, 128}, k in {1, 2, 4, 8}, 16-byte aligned
+// logits): Top-K signatures (Sec. 3.1.1, Eq. 1) with one token per lane.
+//
+// A persistent CTA per SM owns a contiguous range of 32-token tiles.  One
+// producer warp streams each tile [32 tokens x E] into a ring of shared
+// memory slots with 2-D TMA loads (32 x 32 fp32 boxes, 128-byte swizzle, so
+// a lane reading its own row is bank-conflict free); eight consumer warps
+// take the tiles in turn, each lane selecting the Top-K of its token:
+//   1. the row is cut into NG groups of GS consecutive experts and each
+//      group's maximum is kept in registers;
+//   2. K times: a tournament over the group maxima (ties to the lower group)
+//      picks a group, the first element equal to its maximum is selected
+//      (lowest index among equal values), overwritten with -inf in shared
+//      memory, and the group maximum is recomputed.
+// The per-lane selections (a bit per expert) are turned into the signature
+// words of the 32 tokens by 32x32 bit transposes across the warp.
+// The k selected indices of every token are also written (one byte each) for
+// the loss kernel, and the CTAs zero the accumulators of the next kernels.
+#include <climits>
+
+#include "dol_internal.cuh"
+#include "tma.cuh"
+
+namespace dol {
+namespace {
+
+constexpr int kConsumers = 8;
+constexpr int kFastThreads = (kConsumers + 1) * 32;
+constexpr int kBoxBytes = 32 * 128;  // 32 rows x 32 fp32
+
+template <int E>
+struct SigCfg {
+    static constexpr int kBoxes = E / 32;
+    static constexpr int kTileBytes = kBoxes * kBoxBytes;
+    static constexpr int kSlots = (E == 128) ? 12 : 16;
+    static constexpr int GS = (E >= 128) ? E / 16 : 4;  // experts per group
+    static constexpr int NG = E / GS;                    // groups per row
+    static constexpr size_t kSmem = (size_t)kSlots * kTileBytes + 1024 + 2 * kSlots * 8 +
+                                    kSlots * 4 + 16;
+};
+
+// Transpose a 32x32 bit matrix held one row per lane (bit c of lane t is
+// element (t, c)); on return lane c holds column c (bit t = element (t, c)).
+__device__ __forceinline__ uint32_t transpose32(uint32_t x, int lane) {
+    const uint32_t lo_mask[5] = {0x0000FFFFu, 0x00FF00FFu, 0x0F0F0F0Fu, 0x33333333u, 0x55555555u};
+#pragma unroll
+    for (int s = 0; s < 5; ++s) {
+        const int j = 16 >> s;
+        const uint32_t lo = lo_mask[s];
+        const uint32_t p = __shfl_xor_sync(kFull, x, j);
+        x = (lane & j) ? ((x & ~lo) | ((p >> j) & lo)) : ((x & lo) | ((p << j) & ~lo));
+    }
+    return x;
+}
+
+// Byte address of float4 chunk e4 of this lane's row inside a swizzled tile.
+__device__ __forceinline__ unsigned char *chunk_ptr(unsigned char *tile, int e4, int lane) {
+    return tile + (e4 >> 3) * kBoxBytes + lane * 128 + ((((e4 & 7) ^ (lane & 7))) << 4);
+}
+
+template <int K>
+__device__ __forceinline__ void store_idx(uint8_t *p, const int (&sel)[K]) {
+    if (K == 8) {
+        uint2 v;
+        v.x = (uint32_t)sel[0] | ((uint32_t)sel[1 % K] << 8) | ((uint32_t)sel[2 % K] << 16) |
+              ((uint32_t)sel[3 % K] << 24);
+        v.y = (uint32_t)sel[4 % K] | ((uint32_t)sel[5 % K] << 8) | ((uint32_t)sel[6 % K] << 16) |
+              ((uint32_t)sel[7 % K] << 24);
+        *reinterpret_cast<uint2 *>(p) = v;
+    } else if (K == 4) {
+        *reinterpret_cast<uint32_t *>(p) = (uint32_t)sel[0] | ((uint32_t)sel[1 % K] << 8) |
+                                           ((uint32_t)sel[2 % K] << 16) |
+                                           ((uint32_t)sel[3 % K] << 24);
+    } else if (K == 2) {
+        *reinterpret_cast<uint16_t *>(p) = (uint16_t)((uint32_t)sel[0] | ((uint32_t)sel[1 % K] << 8));
+    } else {
+        *p = (uint8_t)sel[0];
+    }
+}
+
+template <int E, int K, bool kCounts>
+__global__ void __launch_bounds__(kFastThreads, 1)
+sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W, int64_t ntiles,
+                uint32_t *__restrict__ bits, int *__restrict__ counts, uint8_t *__restrict__ idx,
+                ZeroSpans zero, int *__restrict__ status) {
+    using C = SigCfg<E>;
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char *smem = reinterpret_cast<unsigned char *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint64_t *full = reinterpret_cast<uint64_t *>(smem + (size_t)C::kSlots * C::kTileBytes);
+    uint64_t *empty = full + C::kSlots;
+    // slot_round[s] = the round of slot s the producer has started to load.
+    // A consumer waits for it before testing the slot's phase parity: the
+    // consumers of consecutive rounds of one slot are different warps, and a
+    // parity test alone cannot tell round r + 1 from round r - 1.
+    volatile int *slot_round = reinterpret_cast<volatile int *>(empty + C::kSlots);
+    volatile int *s_abort = slot_round + C::kSlots;
+
+    pdl_trigger();
+#pragma unroll
+    for (int z = 0; z < 3; ++z)
+        for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < zero.n[z];
+             i += (int64_t)gridDim.x * blockDim.x)
+            zero.p[z][i] = 0;
+
+    const int64_t per = (ntiles + gridDim.x - 1) / gridDim.x;
+    const int64_t tb = (int64_t)blockIdx.x * per;
+    const int64_t te = min64(ntiles, tb + per);
+    const int n = te > tb ? (int)(te - tb) : 0;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < C::kSlots; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+            slot_round[s] = -1;
+        }
+        *s_abort = 0;
+        fence_barrier_init();
+    }
+    __syncthreads();
+
+    if (warp == kConsumers) {  // producer
+        if (lane == 0 && n > 0) {
+            prefetch_tensormap(&tmap);
+            int issued = 0;
+            for (int q = 0; q < n; ++q) {
+                const int s = q % C::kSlots, round = q / C::kSlots;
+                if (round > 0 && !mbar_wait(&empty[s], (round - 1) & 1, status)) {
+                    *s_abort = 1;
+                    break;
+                }
+                if (*s_abort) break;
+                const int64_t tile = tb + q;
+                const int64_t layer = tile / W, w = tile - layer * W;
+                const int y = (int)(layer * T + 32 * w);
+                slot_round[s] = round;
+                mbar_arrive_expect_tx(&full[s], C::kTileBytes);
+#pragma unroll
+                for (int b = 0; b < C::kBoxes; ++b)
+                    tma_load_2d(smem + (size_t)s * C::kTileBytes + b * kBoxBytes, &tmap, b * 32, y,
+                                &full[s]);
+                issued = q + 1;
+            }
+            // Every issued load completes before the CTA may exit.
+            for (int q = issued > C::kSlots ? issued - C::kSlots : 0; q < issued; ++q)
+                mbar_wait(&full[q % C::kSlots], (q / C::kSlots) & 1, status);
+        }
+        return;
+    }
+
+    // consumers
+    constexpr int R = E / 32;
+    constexpr int GS = C::GS, NG = C::NG, GS4 = GS / 4;
+    uint32_t cnt[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) cnt[r] = 0u;
+    int64_t cnt_layer = -1;
+
+    for (int q = warp; q < n; q += kConsumers) {
+        if (*s_abort) break;
+        const int s = q % C::kSlots, round = q / C::kSlots;
+        bool started = slot_round[s] >= round;
+        if (!started) {
+            const unsigned long long t0 = global_ns();
+            while (!(started = slot_round[s] >= round) && !*s_abort) {
+                __nanosleep(64);
+                if (global_ns() - t0 > kWaitLimitNs) {
+                    if (status) atomicOr(status, kDevTimeout);
+                    *s_abort = 1;
+                    break;
+                }
+            }
+        }
+        if (!started || !mbar_wait(&full[s], round & 1, status)) {
+            *s_abort = 1;
+            break;
+        }
+        const int64_t tile = tb + q;
+        const int64_t layer = tile / W, w = tile - layer * W;
+        const int64_t t = 32 * w + lane;
+        const bool valid = t < T;
+        unsigned char *tp = smem + (size_t)s * C::kTileBytes;
+
+        // 1. group maxima
+        float g[NG];
+#pragma unroll
+        for (int gi = 0; gi < NG; ++gi) {
+            float m = -INFINITY;
+#pragma unroll
+            for (int c = 0; c < GS4; ++c) {
+                const float4 v = *reinterpret_cast<const float4 *>(chunk_ptr(tp, gi * GS4 + c, lane));
+                m = fmaxf(m, fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w)));
+            }
+            g[gi] = m;
+        }
+        // 2. K extractions
+        int sel[K];
+#pragma unroll
+        for (int qk = 0; qk < K; ++qk) {
+            float tv[NG];
+            int ti[NG];
+#pragma unroll
+            for (int j = 0; j < NG / 2; ++j) {
+                const bool right = g[2 * j + 1] > g[2 * j];
+                tv[j] = right ? g[2 * j + 1] : g[2 * j];
+                ti[j] = right ? 2 * j + 1 : 2 * j;
+            }
+#pragma unroll
+            for (int nn = NG / 2; nn > 1; nn >>= 1) {
+#pragma unroll
+                for (int j = 0; j < nn / 2; ++j) {
+                    const bool right = tv[2 * j + 1] > tv[2 * j];
+                    tv[j] = right ? tv[2 * j + 1] : tv[2 * j];
+                    ti[j] = right ? ti[2 * j + 1] : ti[2 * j];
+                }
+            }
+            const float bv = tv[0];
+            const int bi = ti[0];
+            float x[GS];
+#pragma unroll
+            for (int c = 0; c < GS4; ++c) {
+                const float4 v = *reinterpret_cast<const float4 *>(chunk_ptr(tp, bi * GS4 + c, lane));
+                x[4 * c] = v.x;
+                x[4 * c + 1] = v.y;
+                x[4 * c + 2] = v.z;
+                x[4 * c + 3] = v.w;
+            }
+            int p = GS - 1;
+#pragma unroll
+            for (int j = GS - 1; j >= 0; --j)
+                if (x[j] == bv) p = j;
+            float m2 = -INFINITY;
+#pragma unroll
+            for (int j = 0; j < GS; ++j) m2 = fmaxf(m2, j == p ? -INFINITY : x[j]);
+            const int e = bi * GS + p;
+            reinterpret_cast<float *>(chunk_ptr(tp, e >> 2, lane))[e & 3] = -INFINITY;
+#pragma unroll
+            for (int gi = 0; gi < NG; ++gi) g[gi] = (gi == bi) ? m2 : g[gi];
+            sel[qk] = e;
+        }
+        // the tile is no longer read: hand the slot back to the producer
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[s]);
+
+        if (idx && valid) store_idx<K>(idx + (layer * T + t) * K, sel);
+        uint32_t m[R];
+#pragma unroll
+        for (int r = 0; r < R; ++r) m[r] = 0u;
+#pragma unroll
+        for (int qk = 0; qk < K; ++qk) {
+            const uint32_t bit = 1u << (sel[qk] & 31);
+            const int rq = sel[qk] >> 5;
+#pragma unroll
+            for (int r = 0; r < R; ++r) m[r] |= (rq == r) ? bit : 0u;
+        }
+        if (kCounts && layer != cnt_layer) {
+            if (cnt_layer >= 0) {
+#pragma unroll
+                for (int r = 0; r < R; ++r)
+                    if (cnt[r]) atomicAdd(&counts[cnt_layer * E + 32 * r + lane], (int)cnt[r]);
+            }
+#pragma unroll
+            for (int r = 0; r < R; ++r) cnt[r] = 0u;
+            cnt_layer = layer;
+        }
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            const uint32_t word = transpose32(valid ? m[r] : 0u, lane);
+            bits[(layer * E + 32 * r + lane) * W + w] = word;
+            if (kCounts) cnt[r] += __popc(word);
+        }
+    }
+    if (kCounts && cnt_layer >= 0) {
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+            if (cnt[r]) atomicAdd(&counts[cnt_layer * E + 32 * r + lane], (int)cnt[r]);
+    }
+}
+
+int sm_count() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 148;
+    return n;
+}
+
+template <int E, int K, bool kCounts>
+cudaError_t run_fast(const CUtensorMap &map, const Problem &p, uint32_t *bits, int *counts,
+                     uint8_t *idx, const ZeroSpans &zero, int *status, cudaStream_t s) {
+    using C = SigCfg<E>;
+    auto kern = sig_fast_kernel<E, K, kCounts>;
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)C::kSmem);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    const int64_t ntiles = (int64_t)p.L * p.W;
+    int64_t grid = sm_count();
+    if (grid > ntiles) grid = ntiles;
+    if (grid < 1) grid = 1;
+    kern<<<(unsigned)grid, kFastThreads, C::kSmem, s>>>(map, p.T, p.W, ntiles, bits, counts, idx,
+                                                        zero, status);
+    return cudaGetLastError();
+}
+
+template <int E, bool kCounts>
+cudaError_t dispatch_k(const CUtensorMap &map, const Problem &p, uint32_t *bits, int *counts,
+                       uint8_t *idx, const ZeroSpans &zero, int *status, cudaStream_t s) {
+    switch (p.k) {
+        case 1: return run_fast<E, 1, kCounts>(map, p, bits, counts, idx, zero, status, s);
+        case 2: return run_fast<E, 2, kCounts>(map, p, bits, counts, idx, zero, status, s);
+        case 4: return run_fast<E, 4, kCounts>(map, p, bits, counts, idx, zero, status, s);
+        default: return run_fast<E, 8, kCounts>(map, p, bits, counts, idx, zero, status, s);
+    }
+}
+
+}  // namespace
+
+bool signatures_fast_supported(const float *logits, const Problem &p) {
+    const bool e_ok = p.E == 32 || p.E == 64 || p.E == 128;
+    const bool k_ok = p.k == 1 || p.k == 2 || p.k == 4 || p.k == 8;
+    return e_ok && k_ok && (reinterpret_cast<uintptr_t>(logits) % 16 == 0) &&
+           (int64_t)p.L * p.T + 32 < (int64_t)INT_MAX;
+}
+
+cudaError_t launch_signatures_fast(const float *logits, const Problem &p, uint32_t *bits,
+                                   int *counts, uint8_t *idx, const ZeroSpans &zero, int *status,
+                                   cudaStream_t s) {
+    CUtensorMap map;
+    if (!encode_tensor_map_2d_f32(&map, logits, (uint64_t)p.L * p.T, (uint64_t)p.E, 32))
+        return cudaErrorInvalidValue;
+    const bool with_counts = counts != nullptr;
+    if (p.E == 32)
+        return with_counts ? dispatch_k<32, true>(map, p, bits, counts, idx, zero, status, s)
+                           : dispatch_k<32, false>(map, p, bits, counts, idx, zero, status, s);
+    if (p.E == 64)
+        return with_counts ? dispatch_k<64, true>(map, p, bits, counts, idx, zero, status, s)
+                           : dispatch_k<64, false>(map, p, bits, counts, idx, zero, status, s);
+    return with_counts ? dispatch_k<128, true>(map, p, bits, counts, idx, zero, status, s)
+                       : dispatch_k<128, false>(map, p, bits, counts, idx, zero, status, s);
+}
+
+}  // namespace dol

@@ -174,3 +174,69 @@ def test_host_entry_point_matches_device_path(dl):
     assert torch.equal(h_dz, dev.dlogits.cpu())
     assert torch.equal(h_counts, dev.counts.cpu())
     assert torch.equal(h_D, dev.D.cpu())
+
+
+@pytest.mark.parametrize(
+    "T,E,k,L,gate,ties",
+    [(1, 128, 8, 1, 0, False), (31, 32, 1, 2, 1, True), (97, 64, 2, 3, 0, True),
+     (1000, 128, 4, 2, 1, False), (4096 + 33, 128, 8, 2, 0, True), (777, 32, 8, 1, 0, False),
+     (3000, 64, 8, 1, 1, True), (2048, 128, 1, 1, 0, True)])
+def test_fast_path_shapes(dl, T, E, k, L, gate, ties):
+    z = workloads.random_logits(T, E, L=L, seed=T + 13 * E + k, ties=ties)
+    out = gpu_run(dl, z, k, gate, grad_scale=3.0)
+    for l in range(L):
+        assert_layer(out, l, z[l].numpy(), k, gate, grad_scale=3.0)
+
+
+def test_fast_and_generic_paths_agree(dl):
+    """A 4-byte-offset view of the same logits takes the generic kernels."""
+    T, E, k = 3000 + 7, 128, 8
+    z = workloads.random_logits(T, E, seed=77, ties=True).cuda()
+    buf = torch.empty(T * E + 1, device="cuda")
+    buf[1:] = z.reshape(-1)
+    zoff = buf[1:].view(1, T, E)
+    assert zoff.data_ptr() % 16 != 0
+    fast = dl.forward_backward(z, k, 0)
+    gen = dl.forward_backward(zoff, k, 0)
+    torch.cuda.synchronize()
+    for name in ("bits", "counts", "D", "origin_do"):
+        assert torch.equal(getattr(fast, name), getattr(gen, name)), name
+    assert float(fast.loss[0]) == pytest.approx(float(gen.loss[0]), rel=1e-5)
+    err = (fast.dlogits - gen.dlogits).abs().max() / gen.dlogits.abs().max()
+    assert float(err) <= 1e-5
+
+
+@pytest.mark.parametrize("E,k,gate", [(128, 8, 0), (64, 2, 1), (32, 4, 0)])
+def test_split_entry_points_fast_path(dl, E, k, gate):
+    T, L = 2500, 2
+    z = workloads.random_logits(T, E, L=L, seed=E + k).cuda()
+    bits, counts = dl.signatures(z, k)
+    D = dl.pairwise_hamming(bits, T)
+    loss, origin, dz = dl.loss_fwd_bwd(z, bits, D, k, gate, grad_scale=0.25)
+    torch.cuda.synchronize()
+    zc = z.cpu()
+    for l in range(L):
+        ref = oracle.forward_backward(zc[l].numpy(), k, gate, grad_scale=0.25)
+        assert np.array_equal(bits[l].cpu().numpy().view(np.uint32), ref["bits"])
+        assert np.array_equal(counts[l].cpu().numpy(), ref["counts"])
+        assert np.array_equal(D[l].cpu().numpy(), ref["D"])
+        assert int(origin[l]) == ref["origin_do"]
+        assert float(loss[l]) == pytest.approx(ref["loss"], rel=LOSS_RTOL)
+        err = np.abs(dz[l].double().cpu().numpy() - ref["dz"]).max() / np.abs(ref["dz"]).max()
+        assert err <= GRAD_TOL
+
+
+def test_repeated_calls_reuse_workspace(dl):
+    """The done counters and partial slots are reused call after call."""
+    w = workloads.get("c3", T=8192)
+    z = workloads.logits(w).cuda()
+    out = dl.Buffers(1, w.T, w.E, w.k, "cuda")
+    first = None
+    for _ in range(5):
+        dl.forward_backward(z, w.k, w.gate, out=out)
+        torch.cuda.synchronize()
+        cur = (out.loss.clone(), out.dlogits.clone(), out.D.clone())
+        if first is None:
+            first = cur
+        assert all(torch.equal(a, b) for a, b in zip(first, cur))
+    assert dl.device_status(out.workspace) == 0
