@@ -92,8 +92,10 @@ do_status do_pairwise_hamming(const uint32_t *bits, int64_t T, int32_t E, int32_
  * (may be NULL for a forward-only call).  bits must hold the selection that
  * produced the token rows of logits; D may come from any source whose row
  * sums fit int32.  workspace: do_workspace_size(T, E, k, L) bytes of device
- * memory, 256-byte aligned, reused across calls; its contents need no
- * initialisation. */
+ * memory, 256-byte aligned and zero-filled before its first use (cudaMemset);
+ * every call leaves it ready for the next one.  A workspace serves one call
+ * at a time; after a call fails or do_device_status reports an error, zero it
+ * again before reusing it. */
 do_status do_loss_fwd_bwd(const float *logits, const uint32_t *bits, const int32_t *D,
                           int64_t T, int32_t E, int32_t k, int32_t L, int32_t gate,
                           float d_scale, float grad_scale, float *loss, int64_t *origin_do,
@@ -120,7 +122,8 @@ do_status do_device_status(void *workspace, void *stream);
  * to the device, runs steps 1-3, and copies loss [L] into h_loss and, when
  * given, dlogits into h_dlogits [L][T][E], counts into h_counts [L][E] and D
  * into h_D [L][E][E].  All device memory comes from `device_buffer`
- * (do_host_buffer_size(T, E, k, L) bytes, 256-byte aligned).  Synchronous:
+ * (do_host_buffer_size(T, E, k, L) bytes, 256-byte aligned, zero-filled
+ * before its first use, as the workspace above).  Synchronous:
  * returns after the results are in host memory and the device status has been
  * checked.  Pinned host memory gives the full copy bandwidth. */
 do_status do_forward_backward_host(const float *h_logits, int64_t T, int32_t E, int32_t k,

@@ -66,7 +66,8 @@ do_status do_signatures(const float *logits, int64_t T, int32_t E, int32_t k, in
         cudaError_t e = cudaMemsetAsync(counts, 0, sizeof(int) * (size_t)p.L * p.E, s);
         const dol::ZeroSpans none = {{nullptr, nullptr, nullptr}, {0, 0, 0}};
         if (e == cudaSuccess)
-            e = dol::launch_signatures_fast(logits, p, bits, counts, nullptr, none, nullptr, s);
+            e = dol::launch_signatures_fast(logits, p, bits, counts, nullptr, nullptr, none, nullptr,
+                                            s);
         return from_cuda(e);
     }
     return from_cuda(dol::launch_signatures(logits, p, bits, counts, s));
@@ -105,9 +106,9 @@ do_status do_loss_fwd_bwd(const float *logits, const uint32_t *bits, const int32
         uint8_t *idx = reinterpret_cast<uint8_t *>(ws + w.idx);
         cudaError_t e = dol::launch_idx_from_bits(bits, p, idx, done, p.L, s);
         if (e == cudaSuccess)
-            e = dol::launch_loss_fast(logits, idx, D, p, gate, d_scale, grad_scale, loss,
-                                      reinterpret_cast<long long *>(origin_do), dlogits,
-                                      reinterpret_cast<double *>(ws + w.partials), done,
+            e = dol::launch_loss_fast(logits, idx, D, nullptr, nullptr, p, gate, d_scale,
+                                      grad_scale, loss, reinterpret_cast<long long *>(origin_do),
+                                      dlogits, reinterpret_cast<double *>(ws + w.partials), done,
                                       reinterpret_cast<int *>(ws), s);
         return from_cuda(e);
     }
@@ -135,19 +136,24 @@ do_status do_forward_backward(const float *logits, int64_t T, int32_t E, int32_t
     cudaStream_t s = (cudaStream_t)stream;
     if (dol::signatures_fast_supported(logits, p) && dol::loss_fast_supported(p, logits, D, dlogits) &&
         aligned(bits, 16)) {
-        // signatures (which clear D, counts and the done counters) -> Hamming -> loss
+        // signatures (+ per-CTA co-occurrence counts) -> reduction to C -> loss,
+        // which builds D = n_i + n_j - 2 c_ij and writes D and the counts
         const dol::WsLayout w = dol::ws_layout(p);
         char *ws = static_cast<char *>(workspace);
         int *done = reinterpret_cast<int *>(ws + w.done);
         uint8_t *idx = reinterpret_cast<uint8_t *>(ws + w.idx);
-        const dol::ZeroSpans zero = {{D, counts, done},
-                                     {(int64_t)p.L * p.E * p.E, (int64_t)p.L * p.E, (int64_t)p.L}};
+        uint32_t *parts = reinterpret_cast<uint32_t *>(ws + w.cooc_parts);
+        int *n_acc = reinterpret_cast<int *>(ws + w.n_acc);
+        const dol::ZeroSpans zero = {{done, nullptr, nullptr}, {(int64_t)p.L, 0, 0}};
         int *status = reinterpret_cast<int *>(ws);
-        cudaError_t e = dol::launch_signatures_fast(logits, p, bits, nullptr, idx, zero, status, s);
-        if (e == cudaSuccess) e = dol::launch_hamming_accumulate(bits, p, D, counts, s);
+        cudaError_t e =
+            dol::launch_signatures_fast(logits, p, bits, n_acc, idx, parts, zero, status, s);
         if (e == cudaSuccess)
-            e = dol::launch_loss_fast(logits, idx, D, p, gate, 1.0f, grad_scale, loss,
-                                      reinterpret_cast<long long *>(origin_do), dlogits,
+            e = dol::launch_cooc_reduce(parts, dol::sig_fast_ctas_per_problem(p), n_acc, p, D,
+                                        counts, s);
+        if (e == cudaSuccess)
+            e = dol::launch_loss_fast(logits, idx, D, counts, n_acc, p, gate, 1.0f, grad_scale,
+                                      loss, reinterpret_cast<long long *>(origin_do), dlogits,
                                       reinterpret_cast<double *>(ws + w.partials), done, status, s);
         return from_cuda(e);
     }

@@ -37,10 +37,16 @@ struct ZeroSpans {
 //   done            [L] int, per-problem count of finished loss CTAs
 //   partials        [L][max CTAs per problem] fp64 sums of A_t
 //   idx             [L][T][k] uint8, the selected experts of every token
+//   cooc_parts      [L][P1][triangle words] uint32, per-CTA co-occurrence counts
+//   n_acc           [L][E] int32, counts summed by the signatures CTAs (kept at
+//                   zero between calls: the loss kernel clears it after use)
 struct WsLayout {
-    size_t done, partials, idx, total;
+    size_t done, partials, idx, cooc_parts, n_acc, total;
     int max_parts;  // partial slots per problem
 };
+// Signatures CTAs per problem on the fast path: min(SMs, kMaxSigCtas) / L.
+constexpr int kMaxSigCtas = 256;
+int max_sig_ctas_per_problem(const Problem &p);
 WsLayout ws_layout(const Problem &p);
 inline size_t workspace_bytes(const Problem &p) { return ws_layout(p).total; }
 
@@ -62,15 +68,32 @@ cudaError_t launch_loss(const float *logits, const uint32_t *bits, const int *D,
 // Fast paths (E in {32, 64, 128}, k in {1, 2, 4, 8}, 16-byte aligned rows).
 bool signatures_fast_supported(const float *logits, const Problem &p);
 cudaError_t launch_signatures_fast(const float *logits, const Problem &p, uint32_t *bits,
-                                   int *counts, uint8_t *idx, const ZeroSpans &zero, int *status,
-                                   cudaStream_t s);
+                                   int *counts, uint8_t *idx, uint32_t *cooc, const ZeroSpans &zero,
+                                   int *status, cudaStream_t s);
 bool loss_fast_supported(const Problem &p, const float *logits, const int *D, const float *dlogits);
 cudaError_t launch_idx_from_bits(const uint32_t *bits, const Problem &p, uint8_t *idx, int *zero_ptr,
                                  int zero_n, cudaStream_t s);
-cudaError_t launch_loss_fast(const float *logits, const uint8_t *idx, const int *D, const Problem &p,
-                             int gate, float d_scale, float grad_scale, float *loss,
-                             long long *origin_do, float *dlogits, double *partials, int *done,
-                             int *status, cudaStream_t s);
+// counts: when given, R_i = (E - 2k) n_i + T k (D local to these tokens) and
+// n_zero ([L][E], may be null) is cleared once D is read; otherwise R_i is a
+// column sum of D.
+cudaError_t launch_loss_fast(const float *logits, const uint8_t *idx, const int *D,
+                             const int *counts, int *n_zero, const Problem &p, int gate,
+                             float d_scale, float grad_scale, float *loss, long long *origin_do,
+                             float *dlogits, double *partials, int *done, int *status,
+                             cudaStream_t s);
+
+// Co-occurrence counts c_ab (a <= b) of one CTA are kept as a triangle whose
+// row a holds columns (a & ~3) .. E-1, so that every row starts 16-byte
+// aligned.  Offset of row a: sum over a' < a of (E - 4 floor(a'/4)).
+template <int E>
+__host__ __device__ constexpr int cooc_row_offset(int a) {
+    return a * E - 8 * (a / 4) * (a / 4 - 1) - 4 * (a % 4) * (a / 4);
+}
+
+int sig_fast_ctas_per_problem(const Problem &p);
+size_t cooc_partial_words(int E);
+cudaError_t launch_cooc_reduce(const uint32_t *partials, int P1, const int *n_acc, const Problem &p,
+                               int *D, int *counts, cudaStream_t s);
 
 // ---------------------------------------------------------------- device helpers
 
@@ -80,6 +103,23 @@ __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
     return v;
+}
+
+// Sum of x[0..n) in a fixed order by a block of nthreads (a power of two):
+// thread i adds x[i], x[i + nthreads], ... in turn, then a fixed tree joins
+// the thread sums.  The result (valid in thread 0) does not depend on timing.
+// red must hold nthreads doubles.  Called by every thread of the block.
+__device__ __forceinline__ double block_sum_fixed(const double *x, int64_t n, double *red,
+                                                  int nthreads) {
+    double s = 0.0;
+    for (int64_t i = threadIdx.x; i < n; i += nthreads) s += __ldcg(x + i);
+    red[threadIdx.x] = s;
+    __syncthreads();
+    for (int o = nthreads / 2; o > 0; o >>= 1) {
+        if ((int)threadIdx.x < o) red[threadIdx.x] += red[threadIdx.x + o];
+        __syncthreads();
+    }
+    return red[0];
 }
 
 __device__ __forceinline__ float warp_max(float v) {

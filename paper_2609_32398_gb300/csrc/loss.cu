@@ -165,11 +165,11 @@ __global__ void __launch_bounds__(256)
 loss_finalize_kernel(const double *__restrict__ partials, int P, const int *__restrict__ Dg, int E,
                      double scale, float *__restrict__ loss, long long *__restrict__ origin_do) {
     __shared__ long long s_red[256];
+    __shared__ double s_dred[256];
     const int layer = blockIdx.x;
-    if (threadIdx.x == 0) {
-        double s = 0.0;
-        for (int b = 0; b < P; ++b) s += partials[(int64_t)layer * P + b];
-        loss[layer] = (float)(s * scale);
+    {
+        const double s = block_sum_fixed(partials + (int64_t)layer * P, P, s_dred, 256);
+        if (threadIdx.x == 0) loss[layer] = (float)(s * scale);
     }
     if (origin_do) {
         const int *Dl = Dg + (int64_t)layer * E * E;
@@ -237,11 +237,24 @@ WsLayout ws_layout(const Problem &p) {
     const int64_t gen_parts = loss_blocks_per_problem(p);
     w.max_parts = (int)(fast_parts > gen_parts ? fast_parts : gen_parts);
     const bool fast_k = p.k == 1 || p.k == 2 || p.k == 4 || p.k == 8;
+    const bool fast_e = p.E == 32 || p.E == 64 || p.E == 128;
     w.done = kWsHeader;
     w.partials = up(w.done + sizeof(int) * (size_t)p.L);
     w.idx = up(w.partials + sizeof(double) * (size_t)p.L * (size_t)w.max_parts);
-    w.total = up(w.idx + (fast_k ? (size_t)p.L * (size_t)p.T * (size_t)p.k : 0));
+    w.cooc_parts = up(w.idx + (fast_k ? (size_t)p.L * (size_t)p.T * (size_t)p.k : 0));
+    const size_t parts = (fast_k && fast_e) ? sizeof(uint32_t) * (size_t)p.L *
+                                                  (size_t)max_sig_ctas_per_problem(p) *
+                                                  cooc_partial_words(p.E)
+                                            : 0;
+    w.n_acc = up(w.cooc_parts + parts);
+    w.total = up(w.n_acc + ((fast_k && fast_e) ? sizeof(int) * (size_t)p.L * p.E : 0));
     return w;
+}
+
+int max_sig_ctas_per_problem(const Problem &p) {
+    int64_t gx = kMaxSigCtas / p.L;
+    if (gx > p.W) gx = p.W;
+    return (int)(gx < 1 ? 1 : gx);
 }
 
 cudaError_t launch_loss(const float *logits, const uint32_t *bits, const int *D, const Problem &p,

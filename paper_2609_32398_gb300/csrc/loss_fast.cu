@@ -9,11 +9,16 @@
 // gives every w_it without looking at the signature bits.  D must be
 // symmetric (every Hamming matrix and every sum of them is).
 //
-// Layout: a CTA copies D into shared memory once (bulk copy), writes the
-// diagonal -R_i, then its warps walk tokens with G = E/16 lanes per token;
-// lane g of a token group owns experts c*E/4 + 4g .. +3 for c = 0..3, so the
-// group reads 16-byte chunks of the logits row, of the D' rows and writes the
-// dlogits row with coalesced 16-byte accesses.  Per token:
+// R_i is a column sum of D, or -- in the fused path, where D comes from the
+// same tokens' co-occurrence counts (D_ij = n_i + n_j - 2 c_ij, App. C.3) --
+//   R_i = (E - 2k) n_i + T k      (sum_j c_ij = k n_i, sum_j n_j = T k).
+//
+// Layout: a CTA stages D' in shared memory, then its warps walk tokens with
+// G = E/16 lanes per token; lane g of a token group owns experts
+// c*E/4 + 4g .. +3 for c = 0..3, so a group reads 16-byte chunks of the
+// logits row and of the D' rows and writes the dlogits row with coalesced
+// 16-byte accesses.  The next token group's logits and indices are loaded
+// while the current one is computed.  Per token:
 //   sigmoid-norm  s = sigmoid(z), A = sum s w / sum s,
 //                 dz = c s (1 - s) (w - A) / sum s
 //   softmax       e = exp(z - max), A = sum e w / sum e, dz = c e (w - A) / sum e
@@ -57,65 +62,127 @@ __device__ __forceinline__ void load_idx(const uint8_t *p, int (&j)[K]) {
     }
 }
 
-template <int E, int K, int kGate>
+struct LossArgs {
+    const float *logits;
+    const uint8_t *idx;
+    const int *D;        // [L][E][E], symmetric
+    const int *counts;   // fused path: n_i [L][E] of the same tokens (else null)
+    int *n_zero;         // fused path: accumulator [L][E] to clear after use (or null)
+    int64_t T;
+    int k;
+    int tokens_per_cta;
+    float coef;
+    double scale;
+    float *dlogits;
+    double *partials;
+    int *done;
+    float *loss;
+    long long *origin_do;
+    int *status;
+};
+
+template <int E, int K, int kGate, bool kRFromCounts>
 __global__ void __launch_bounds__(kLossFastThreads)
-loss_fast_kernel(const float *__restrict__ logits, const uint8_t *__restrict__ idx,
-                 const int *__restrict__ Dg, int64_t T, int tokens_per_cta, float coef,
-                 double scale, float *__restrict__ dlogits, double *__restrict__ partials,
-                 int *__restrict__ done, float *__restrict__ loss, long long *__restrict__ origin_do,
-                 int *__restrict__ status) {
-    constexpr int G = E / 16;       // lanes per token
-    constexpr int TPW = 32 / G;     // tokens per warp pass
-    constexpr int Q = E / 4;        // expert stride between a lane's chunks
+loss_fast_kernel(const LossArgs a) {
+    constexpr int G = E / 16;    // lanes per token
+    constexpr int TPW = 32 / G;  // tokens per warp pass
+    constexpr int Q = E / 4;     // expert stride between a lane's chunks
     extern __shared__ __align__(128) int sD[];  // [E][E]
     __shared__ __align__(8) uint64_t bar;
     __shared__ double s_part[kLossFastWarps];
+    __shared__ long long s_o[kLossFastWarps];
+    __shared__ long long s_r[E];
     __shared__ int s_last;
 
     const int layer = blockIdx.y;
     const int P = gridDim.x;
-    const int *Dl = Dg + (int64_t)layer * E * E;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int grp = lane / G, g = lane % G;
+    const int64_t T = a.T;
+    const float *zl = a.logits + (int64_t)layer * T * E;
+    float *dzl = a.dlogits ? a.dlogits + (int64_t)layer * T * E : nullptr;
+    const uint8_t *il = a.idx + (int64_t)layer * T * K;
+    const int64_t t_begin = (int64_t)blockIdx.x * a.tokens_per_cta;
+    const int64_t t_end = min64(T, t_begin + a.tokens_per_cta);
+    const int64_t stride = (int64_t)kLossFastWarps * TPW;
 
     if (threadIdx.x == 0) {
         mbar_init(&bar, 1);
         fence_barrier_init();
     }
-    __syncthreads();
-    pdl_wait();  // D, idx and the zeroed counters come from the previous kernels
-    if (threadIdx.x == 0) {
-        mbar_arrive_expect_tx(&bar, (uint32_t)(sizeof(int) * E * E));
-        bulk_load(sD, Dl, (uint32_t)(sizeof(int) * E * E), &bar);
-    }
-    const bool have_d = mbar_wait(&bar, 0, status);
-    if (__syncthreads_or(!have_d)) return;
-    if (threadIdx.x < E) {
-        const int i = threadIdx.x;
-        long long r = 0;
-        for (int j = 0; j < E; ++j) r += sD[j * E + i];
-        if (r > INT_MAX || r < 0) atomicOr(status, kDevOverflow);
-        sD[i * E + i] = -(int)r;
-    }
-    __syncthreads();
-
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int grp = lane / G, g = lane % G;
-    const float *zl = logits + (int64_t)layer * T * E;
-    float *dzl = dlogits ? dlogits + (int64_t)layer * T * E : nullptr;
-    const uint8_t *il = idx + (int64_t)layer * T * K;
-    const int64_t t_begin = (int64_t)blockIdx.x * tokens_per_cta;
-    const int64_t t_end = min64(T, t_begin + tokens_per_cta);
-    double tok_sum = 0.0;
-
-    for (int64_t tb = t_begin + (int64_t)warp * TPW; tb < t_end; tb += (int64_t)kLossFastWarps * TPW) {
+    // The logits are an input of the whole path, so the first token group's
+    // rows can be fetched before the previous kernels have finished.
+    int64_t tb = t_begin + (int64_t)warp * TPW;
+    float4 zc[4];
+    {
         const int64_t t = tb + grp;
-        const bool valid = t < t_end;
-        const int64_t tc = valid ? t : t_begin;  // clamp: invalid lanes recompute a valid token
-        int js[K];
-        load_idx<K>(il + tc * K, js);
-        float4 zc[4];
+        const int64_t tc = (t < t_end) ? t : t_begin;
 #pragma unroll
         for (int c = 0; c < 4; ++c)
             zc[c] = __ldg(reinterpret_cast<const float4 *>(zl + tc * E + c * Q + 4 * g));
+    }
+    __syncthreads();
+    pdl_wait();  // D, idx and the cleared counters come from the previous kernels
+    if (threadIdx.x == 0) {
+        mbar_arrive_expect_tx(&bar, (uint32_t)(sizeof(int) * E * E));
+        bulk_load(sD, a.D + (int64_t)layer * E * E, (uint32_t)(sizeof(int) * E * E), &bar);
+    }
+    int js[K];
+    {
+        const int64_t t = tb + grp;
+        load_idx<K>(il + ((t < t_end) ? t : t_begin) * K, js);
+    }
+    const bool have_d = mbar_wait(&bar, 0, a.status);
+    if (__syncthreads_or(!have_d)) return;
+
+    if (kRFromCounts) {
+        if (threadIdx.x < E) {
+            const int i = threadIdx.x;
+            const long long n = a.counts[(int64_t)layer * E + i];
+            const long long r = (long long)(E - 2 * K) * n + T * (long long)K;
+            if (r > INT_MAX || r < 0) atomicOr(a.status, kDevOverflow);
+            sD[i * E + i] = -(int)r;
+            if (a.n_zero && blockIdx.x == 0) a.n_zero[(int64_t)layer * E + i] = 0;
+        }
+    } else {
+        // R_i = sum_j D_ji (D symmetric): kPer threads per column, four chains each
+        constexpr int kPer = kLossFastThreads / E;  // 2, 4 or 8
+        const int i = threadIdx.x % E, part = threadIdx.x / E;
+        long long r0 = 0, r1 = 0, r2 = 0, r3 = 0;
+        for (int j = part; j < E; j += 4 * kPer) {
+            r0 += sD[j * E + i];
+            if (j + kPer < E) r1 += sD[(j + kPer) * E + i];
+            if (j + 2 * kPer < E) r2 += sD[(j + 2 * kPer) * E + i];
+            if (j + 3 * kPer < E) r3 += sD[(j + 3 * kPer) * E + i];
+        }
+        if (threadIdx.x < E) s_r[threadIdx.x] = 0;
+        __syncthreads();
+        atomicAdd(reinterpret_cast<unsigned long long *>(&s_r[i]),
+                  (unsigned long long)(r0 + r1 + r2 + r3));
+        __syncthreads();
+        if (threadIdx.x < E) {
+            const long long r = s_r[threadIdx.x];
+            if (r > INT_MAX || r < 0) atomicOr(a.status, kDevOverflow);
+            sD[threadIdx.x * E + threadIdx.x] = -(int)r;
+        }
+    }
+    __syncthreads();
+
+    double tok_sum = 0.0;
+    for (; tb < t_end; tb += stride) {
+        const int64_t t = tb + grp;
+        const bool valid = t < t_end;
+        // prefetch the next token group
+        const int64_t tn = tb + stride + grp;
+        const int64_t tnc = (tn < t_end) ? tn : t_begin;
+        float4 zn[4];
+        int jn[K];
+        if (tb + stride < t_end) {
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                zn[c] = __ldg(reinterpret_cast<const float4 *>(zl + tnc * E + c * Q + 4 * g));
+            load_idx<K>(il + tnc * K, jn);
+        }
         int4 acc[4];
 #pragma unroll
         for (int c = 0; c < 4; ++c) acc[c] = make_int4(0, 0, 0, 0);
@@ -173,7 +240,7 @@ loss_fast_kernel(const float *__restrict__ logits, const uint8_t *__restrict__ i
         const float A = num * inv;
         if (valid && g == 0) tok_sum += (double)A;
         if (dzl && valid) {
-            const float cs = coef * inv;
+            const float cs = a.coef * inv;
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 float4 o;
@@ -187,6 +254,10 @@ loss_fast_kernel(const float *__restrict__ logits, const uint8_t *__restrict__ i
                 *reinterpret_cast<float4 *>(dzl + t * E + c * Q + 4 * g) = o;
             }
         }
+#pragma unroll
+        for (int c = 0; c < 4; ++c) zc[c] = zn[c];
+#pragma unroll
+        for (int q = 0; q < K; ++q) js[q] = jn[q];
     }
     // CTA partial, in warp and lane order
 #pragma unroll
@@ -196,22 +267,24 @@ loss_fast_kernel(const float *__restrict__ logits, const uint8_t *__restrict__ i
     if (threadIdx.x == 0) {
         double sum = 0.0;
         for (int q = 0; q < kLossFastWarps; ++q) sum += s_part[q];
-        partials[(int64_t)layer * P + blockIdx.x] = sum;
+        a.partials[(int64_t)layer * P + blockIdx.x] = sum;
         __threadfence();
-        s_last = (atomicAdd(&done[layer], 1) == P - 1);
+        s_last = (atomicAdd(&a.done[layer], 1) == P - 1);
     }
     __syncthreads();
     if (!s_last) return;
     // last CTA of this problem: fixed-order sum of the partials, origin_do
     __threadfence();
-    if (threadIdx.x == 0) {
-        const volatile double *pp = partials + (int64_t)layer * P;
-        double sum = 0.0;
-        for (int b = 0; b < P; ++b) sum += pp[b];
-        loss[layer] = (float)(sum * scale);
-        done[layer] = 0;
+    {
+        __shared__ double s_red[kLossFastThreads];
+        const double sum = block_sum_fixed(a.partials + (int64_t)layer * P, P, s_red,
+                                           kLossFastThreads);
+        if (threadIdx.x == 0) {
+            a.loss[layer] = (float)(sum * a.scale);
+            a.done[layer] = 0;
+        }
     }
-    if (origin_do) {
+    if (a.origin_do) {
         long long o = 0;
         for (int e = threadIdx.x; e < E * E; e += blockDim.x) {
             const int i = e / E, j = e - (e / E) * E;
@@ -222,13 +295,12 @@ loss_fast_kernel(const float *__restrict__ logits, const uint8_t *__restrict__ i
         }
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) o += __shfl_xor_sync(kFull, o, off);
-        __shared__ long long s_o[kLossFastWarps];
         if (lane == 0) s_o[warp] = o;
         __syncthreads();
         if (threadIdx.x == 0) {
             long long sum = 0;
             for (int q = 0; q < kLossFastWarps; ++q) sum += s_o[q];
-            origin_do[layer] = sum;
+            a.origin_do[layer] = sum;
         }
     }
 }
@@ -288,18 +360,15 @@ idx_from_bits_kernel(const uint32_t *__restrict__ bits, int64_t T, int64_t W, in
     }
 }
 
-template <int E, int K>
-cudaError_t run_loss_fast(const float *logits, const uint8_t *idx, const int *D, const Problem &p,
-                          int gate, float coef, double scale, float *dlogits, double *partials,
-                          int P, int tokens_per_cta, int *done, float *loss, long long *origin_do,
-                          int *status, cudaStream_t s) {
+template <int E, int K, bool kRFromCounts>
+cudaError_t run_loss_fast(const LossArgs &args, int gate, int P, const Problem &p, cudaStream_t s) {
     const size_t smem = sizeof(int) * E * E;
     static bool attr_set = false;
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(loss_fast_kernel<E, K, 0>,
+        cudaError_t e = cudaFuncSetAttribute(loss_fast_kernel<E, K, 0, kRFromCounts>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(loss_fast_kernel<E, K, 1>,
+            e = cudaFuncSetAttribute(loss_fast_kernel<E, K, 1, kRFromCounts>,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         attr_set = true;
@@ -314,23 +383,17 @@ cudaError_t run_loss_fast(const float *logits, const uint8_t *idx, const int *D,
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    if (gate == 0)
-        return cudaLaunchKernelEx(&cfg, loss_fast_kernel<E, K, 0>, logits, idx, D, p.T, tokens_per_cta,
-                                  coef, scale, dlogits, partials, done, loss, origin_do, status);
-    return cudaLaunchKernelEx(&cfg, loss_fast_kernel<E, K, 1>, logits, idx, D, p.T, tokens_per_cta,
-                              coef, scale, dlogits, partials, done, loss, origin_do, status);
+    if (gate == 0) return cudaLaunchKernelEx(&cfg, loss_fast_kernel<E, K, 0, kRFromCounts>, args);
+    return cudaLaunchKernelEx(&cfg, loss_fast_kernel<E, K, 1, kRFromCounts>, args);
 }
 
-template <int E>
-cudaError_t dispatch_loss_k(const float *logits, const uint8_t *idx, const int *D, const Problem &p,
-                            int gate, float coef, double scale, float *dlogits, double *partials,
-                            int P, int tpc, int *done, float *loss, long long *origin_do, int *status,
-                            cudaStream_t s) {
+template <int E, bool kRFromCounts>
+cudaError_t dispatch_loss_k(const LossArgs &args, int gate, int P, const Problem &p, cudaStream_t s) {
     switch (p.k) {
-        case 1: return run_loss_fast<E, 1>(logits, idx, D, p, gate, coef, scale, dlogits, partials, P, tpc, done, loss, origin_do, status, s);
-        case 2: return run_loss_fast<E, 2>(logits, idx, D, p, gate, coef, scale, dlogits, partials, P, tpc, done, loss, origin_do, status, s);
-        case 4: return run_loss_fast<E, 4>(logits, idx, D, p, gate, coef, scale, dlogits, partials, P, tpc, done, loss, origin_do, status, s);
-        default: return run_loss_fast<E, 8>(logits, idx, D, p, gate, coef, scale, dlogits, partials, P, tpc, done, loss, origin_do, status, s);
+        case 1: return run_loss_fast<E, 1, kRFromCounts>(args, gate, P, p, s);
+        case 2: return run_loss_fast<E, 2, kRFromCounts>(args, gate, P, p, s);
+        case 4: return run_loss_fast<E, 4, kRFromCounts>(args, gate, P, p, s);
+        default: return run_loss_fast<E, 8, kRFromCounts>(args, gate, P, p, s);
     }
 }
 
@@ -360,7 +423,7 @@ void loss_fast_grid(const Problem &p, int *P, int *tokens_per_cta) {
     int dev = 0, sms = 148;
     if (cudaGetDevice(&dev) == cudaSuccess)
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    int64_t want = (int64_t)sms * 3 / p.L;
+    int64_t want = (int64_t)sms * 2 / p.L;  // two CTAs fit on an SM: one wave
     if (want < 1) want = 1;
     int64_t tpc = (p.T + want - 1) / want;
     tpc = (tpc + 31) / 32 * 32;
@@ -387,20 +450,39 @@ cudaError_t launch_idx_from_bits(const uint32_t *bits, const Problem &p, uint8_t
     return cudaErrorInvalidValue;
 }
 
-cudaError_t launch_loss_fast(const float *logits, const uint8_t *idx, const int *D, const Problem &p,
-                             int gate, float d_scale, float grad_scale, float *loss,
-                             long long *origin_do, float *dlogits, double *partials, int *done,
-                             int *status, cudaStream_t s) {
+cudaError_t launch_loss_fast(const float *logits, const uint8_t *idx, const int *D,
+                             const int *counts, int *n_zero, const Problem &p, int gate,
+                             float d_scale, float grad_scale, float *loss, long long *origin_do,
+                             float *dlogits, double *partials, int *done, int *status,
+                             cudaStream_t s) {
     int P = 1, tpc = 32;
     loss_fast_grid(p, &P, &tpc);
     const double norm = 1.0 / ((double)p.T * (double)p.T * (double)p.k);
-    const float coef = (float)((double)grad_scale * (double)d_scale * norm);
-    const double scale = (double)d_scale * norm;
-    if (p.E == 32)
-        return dispatch_loss_k<32>(logits, idx, D, p, gate, coef, scale, dlogits, partials, P, tpc, done, loss, origin_do, status, s);
-    if (p.E == 64)
-        return dispatch_loss_k<64>(logits, idx, D, p, gate, coef, scale, dlogits, partials, P, tpc, done, loss, origin_do, status, s);
-    return dispatch_loss_k<128>(logits, idx, D, p, gate, coef, scale, dlogits, partials, P, tpc, done, loss, origin_do, status, s);
+    LossArgs args;
+    args.logits = logits;
+    args.idx = idx;
+    args.D = D;
+    args.counts = counts;
+    args.n_zero = n_zero;
+    args.T = p.T;
+    args.k = p.k;
+    args.tokens_per_cta = tpc;
+    args.coef = (float)((double)grad_scale * (double)d_scale * norm);
+    args.scale = (double)d_scale * norm;
+    args.dlogits = dlogits;
+    args.partials = partials;
+    args.done = done;
+    args.loss = loss;
+    args.origin_do = origin_do;
+    args.status = status;
+    if (counts) {
+        if (p.E == 32) return dispatch_loss_k<32, true>(args, gate, P, p, s);
+        if (p.E == 64) return dispatch_loss_k<64, true>(args, gate, P, p, s);
+        return dispatch_loss_k<128, true>(args, gate, P, p, s);
+    }
+    if (p.E == 32) return dispatch_loss_k<32, false>(args, gate, P, p, s);
+    if (p.E == 64) return dispatch_loss_k<64, false>(args, gate, P, p, s);
+    return dispatch_loss_k<128, false>(args, gate, P, p, s);
 }
 
 }  // namespace dol

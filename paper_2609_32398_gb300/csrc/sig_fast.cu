@@ -32,12 +32,15 @@ template <int E>
 struct SigCfg {
     static constexpr int kBoxes = E / 32;
     static constexpr int kTileBytes = kBoxes * kBoxBytes;
-    static constexpr int kSlots = (E == 128) ? 12 : 16;
+    static constexpr int kSlots = (E == 128) ? 11 : 16;
     static constexpr int GS = (E >= 128) ? E / 16 : 4;  // experts per group
     static constexpr int NG = E / GS;                    // groups per row
+    // co-occurrence counters: row a holds columns (a & ~3) .. E-1
+    static constexpr int kCoocWords = cooc_row_offset<E>(E);
     static constexpr size_t kSmem = (size_t)kSlots * kTileBytes + 1024 + 2 * kSlots * 8 +
-                                    kSlots * 4 + 16;
+                                    kSlots * 4 + 32 + (size_t)kCoocWords * 4 + E * 4;
 };
+
 
 // Transpose a 32x32 bit matrix held one row per lane (bit c of lane t is
 // element (t, c)); on return lane c holds column c (bit t = element (t, c)).
@@ -78,11 +81,11 @@ __device__ __forceinline__ void store_idx(uint8_t *p, const int (&sel)[K]) {
     }
 }
 
-template <int E, int K, bool kCounts>
+template <int E, int K, bool kCounts, bool kCooc>
 __global__ void __launch_bounds__(kFastThreads, 1)
-sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W, int64_t ntiles,
+sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W,
                 uint32_t *__restrict__ bits, int *__restrict__ counts, uint8_t *__restrict__ idx,
-                ZeroSpans zero, int *__restrict__ status) {
+                uint32_t *__restrict__ cooc, ZeroSpans zero, int *__restrict__ status) {
     using C = SigCfg<E>;
     extern __shared__ unsigned char smem_raw[];
     unsigned char *smem = reinterpret_cast<unsigned char *>(
@@ -95,6 +98,9 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W, 
     // parity test alone cannot tell round r + 1 from round r - 1.
     volatile int *slot_round = reinterpret_cast<volatile int *>(empty + C::kSlots);
     volatile int *s_abort = slot_round + C::kSlots;
+    uint32_t *s_cooc = reinterpret_cast<uint32_t *>(
+        (reinterpret_cast<uintptr_t>(s_abort + 1) + 15) & ~uintptr_t(15));
+    int *s_rowoff = reinterpret_cast<int *>(s_cooc + C::kCoocWords);
 
     pdl_trigger();
 #pragma unroll
@@ -103,11 +109,17 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W, 
              i += (int64_t)gridDim.x * blockDim.x)
             zero.p[z][i] = 0;
 
-    const int64_t per = (ntiles + gridDim.x - 1) / gridDim.x;
+    // this CTA: layer blockIdx.y, a contiguous range of its 32-token tiles
+    const int64_t layer = blockIdx.y;
+    const int64_t per = (W + gridDim.x - 1) / gridDim.x;
     const int64_t tb = (int64_t)blockIdx.x * per;
-    const int64_t te = min64(ntiles, tb + per);
+    const int64_t te = min64(W, tb + per);
     const int n = te > tb ? (int)(te - tb) : 0;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (kCooc) {
+        for (int i = threadIdx.x; i < C::kCoocWords; i += blockDim.x) s_cooc[i] = 0u;
+        for (int a = threadIdx.x; a < E; a += blockDim.x) s_rowoff[a] = cooc_row_offset<E>(a) - (a & ~3);
+    }
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < C::kSlots; ++s) {
@@ -131,8 +143,7 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W, 
                     break;
                 }
                 if (*s_abort) break;
-                const int64_t tile = tb + q;
-                const int64_t layer = tile / W, w = tile - layer * W;
+                const int64_t w = tb + q;
                 const int y = (int)(layer * T + 32 * w);
                 slot_round[s] = round;
                 mbar_arrive_expect_tx(&full[s], C::kTileBytes);
@@ -155,7 +166,6 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W, 
     uint32_t cnt[R];
 #pragma unroll
     for (int r = 0; r < R; ++r) cnt[r] = 0u;
-    int64_t cnt_layer = -1;
 
     for (int q = warp; q < n; q += kConsumers) {
         if (*s_abort) break;
@@ -176,8 +186,7 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W, 
             *s_abort = 1;
             break;
         }
-        const int64_t tile = tb + q;
-        const int64_t layer = tile / W, w = tile - layer * W;
+        const int64_t w = tb + q;
         const int64_t t = 32 * w + lane;
         const bool valid = t < T;
         unsigned char *tp = smem + (size_t)s * C::kTileBytes;
@@ -245,6 +254,16 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W, 
         if (lane == 0) mbar_arrive(&empty[s]);
 
         if (idx && valid) store_idx<K>(idx + (layer * T + t) * K, sel);
+        if (kCooc && valid) {
+            // c_ab += 1 for every pair a <= b of selected experts (a = b gives n_a)
+#pragma unroll
+            for (int q1 = 0; q1 < K; ++q1)
+#pragma unroll
+                for (int q2 = q1; q2 < K; ++q2) {
+                    const int a = min(sel[q1], sel[q2]), b = max(sel[q1], sel[q2]);
+                    atomicAdd(&s_cooc[s_rowoff[a] + b], 1u);
+                }
+        }
         uint32_t m[R];
 #pragma unroll
         for (int r = 0; r < R; ++r) m[r] = 0u;
@@ -255,16 +274,6 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W, 
 #pragma unroll
             for (int r = 0; r < R; ++r) m[r] |= (rq == r) ? bit : 0u;
         }
-        if (kCounts && layer != cnt_layer) {
-            if (cnt_layer >= 0) {
-#pragma unroll
-                for (int r = 0; r < R; ++r)
-                    if (cnt[r]) atomicAdd(&counts[cnt_layer * E + 32 * r + lane], (int)cnt[r]);
-            }
-#pragma unroll
-            for (int r = 0; r < R; ++r) cnt[r] = 0u;
-            cnt_layer = layer;
-        }
 #pragma unroll
         for (int r = 0; r < R; ++r) {
             const uint32_t word = transpose32(valid ? m[r] : 0u, lane);
@@ -272,10 +281,25 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W, 
             if (kCounts) cnt[r] += __popc(word);
         }
     }
-    if (kCounts && cnt_layer >= 0) {
+    if (kCounts) {
 #pragma unroll
         for (int r = 0; r < R; ++r)
-            if (cnt[r]) atomicAdd(&counts[cnt_layer * E + 32 * r + lane], (int)cnt[r]);
+            if (cnt[r]) atomicAdd(&counts[layer * E + 32 * r + lane], (int)cnt[r]);
+    }
+    if (kCooc) {
+        // all consumer warps have counted: store this CTA's triangle for the
+        // reduction kernel
+        asm volatile("bar.sync 1, %0;" ::"n"(kConsumers * 32) : "memory");
+        uint4 *dst = reinterpret_cast<uint4 *>(cooc + ((size_t)layer * gridDim.x + blockIdx.x) *
+                                                          (size_t)C::kCoocWords);
+        const uint4 *src = reinterpret_cast<const uint4 *>(s_cooc);
+        for (int i = threadIdx.x; i < C::kCoocWords / 4; i += kConsumers * 32) dst[i] = src[i];
+        // the diagonal holds this CTA's counts n_a: add them to the layer's totals
+        // (counts points at the workspace accumulator on this path)
+        for (int a = threadIdx.x; a < E; a += kConsumers * 32) {
+            const uint32_t na = s_cooc[s_rowoff[a] + a];
+            if (na) atomicAdd(&counts[layer * E + a], (int)na);
+        }
     }
 }
 
@@ -286,11 +310,12 @@ int sm_count() {
     return n;
 }
 
-template <int E, int K, bool kCounts>
+template <int E, int K, bool kCounts, bool kCooc>
 cudaError_t run_fast(const CUtensorMap &map, const Problem &p, uint32_t *bits, int *counts,
-                     uint8_t *idx, const ZeroSpans &zero, int *status, cudaStream_t s) {
+                     uint8_t *idx, uint32_t *cooc, const ZeroSpans &zero, int *status,
+                     cudaStream_t s) {
     using C = SigCfg<E>;
-    auto kern = sig_fast_kernel<E, K, kCounts>;
+    auto kern = sig_fast_kernel<E, K, kCounts, kCooc>;
     static bool attr_set = false;
     if (!attr_set) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -298,27 +323,46 @@ cudaError_t run_fast(const CUtensorMap &map, const Problem &p, uint32_t *bits, i
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    const int64_t ntiles = (int64_t)p.L * p.W;
-    int64_t grid = sm_count();
-    if (grid > ntiles) grid = ntiles;
-    if (grid < 1) grid = 1;
-    kern<<<(unsigned)grid, kFastThreads, C::kSmem, s>>>(map, p.T, p.W, ntiles, bits, counts, idx,
-                                                        zero, status);
+    dim3 grid((unsigned)sig_fast_ctas_per_problem(p), (unsigned)p.L);
+    kern<<<grid, kFastThreads, C::kSmem, s>>>(map, p.T, p.W, bits, counts, idx, cooc, zero, status);
     return cudaGetLastError();
 }
 
-template <int E, bool kCounts>
+template <int E, bool kCounts, bool kCooc>
 cudaError_t dispatch_k(const CUtensorMap &map, const Problem &p, uint32_t *bits, int *counts,
-                       uint8_t *idx, const ZeroSpans &zero, int *status, cudaStream_t s) {
+                       uint8_t *idx, uint32_t *cooc, const ZeroSpans &zero, int *status,
+                       cudaStream_t s) {
     switch (p.k) {
-        case 1: return run_fast<E, 1, kCounts>(map, p, bits, counts, idx, zero, status, s);
-        case 2: return run_fast<E, 2, kCounts>(map, p, bits, counts, idx, zero, status, s);
-        case 4: return run_fast<E, 4, kCounts>(map, p, bits, counts, idx, zero, status, s);
-        default: return run_fast<E, 8, kCounts>(map, p, bits, counts, idx, zero, status, s);
+        case 1: return run_fast<E, 1, kCounts, kCooc>(map, p, bits, counts, idx, cooc, zero, status, s);
+        case 2: return run_fast<E, 2, kCounts, kCooc>(map, p, bits, counts, idx, cooc, zero, status, s);
+        case 4: return run_fast<E, 4, kCounts, kCooc>(map, p, bits, counts, idx, cooc, zero, status, s);
+        default: return run_fast<E, 8, kCounts, kCooc>(map, p, bits, counts, idx, cooc, zero, status, s);
     }
 }
 
+template <int E>
+cudaError_t dispatch_mode(const CUtensorMap &map, const Problem &p, uint32_t *bits, int *counts,
+                          uint8_t *idx, uint32_t *cooc, const ZeroSpans &zero, int *status,
+                          cudaStream_t s) {
+    // split entry point: counts, no co-occurrence; fused path: co-occurrence
+    if (cooc) return dispatch_k<E, false, true>(map, p, bits, counts, idx, cooc, zero, status, s);
+    return dispatch_k<E, true, false>(map, p, bits, counts, idx, cooc, zero, status, s);
+}
+
 }  // namespace
+
+int sig_fast_ctas_per_problem(const Problem &p) {
+    int sms = sm_count();
+    if (sms > kMaxSigCtas) sms = kMaxSigCtas;
+    int64_t gx = sms / p.L;
+    if (gx > p.W) gx = p.W;
+    if (gx < 1) gx = 1;
+    return (int)gx;
+}
+
+size_t cooc_partial_words(int E) {
+    return E == 32 ? SigCfg<32>::kCoocWords : E == 64 ? SigCfg<64>::kCoocWords : SigCfg<128>::kCoocWords;
+}
 
 bool signatures_fast_supported(const float *logits, const Problem &p) {
     const bool e_ok = p.E == 32 || p.E == 64 || p.E == 128;
@@ -328,20 +372,14 @@ bool signatures_fast_supported(const float *logits, const Problem &p) {
 }
 
 cudaError_t launch_signatures_fast(const float *logits, const Problem &p, uint32_t *bits,
-                                   int *counts, uint8_t *idx, const ZeroSpans &zero, int *status,
-                                   cudaStream_t s) {
+                                   int *counts, uint8_t *idx, uint32_t *cooc, const ZeroSpans &zero,
+                                   int *status, cudaStream_t s) {
     CUtensorMap map;
     if (!encode_tensor_map_2d_f32(&map, logits, (uint64_t)p.L * p.T, (uint64_t)p.E, 32))
         return cudaErrorInvalidValue;
-    const bool with_counts = counts != nullptr;
-    if (p.E == 32)
-        return with_counts ? dispatch_k<32, true>(map, p, bits, counts, idx, zero, status, s)
-                           : dispatch_k<32, false>(map, p, bits, counts, idx, zero, status, s);
-    if (p.E == 64)
-        return with_counts ? dispatch_k<64, true>(map, p, bits, counts, idx, zero, status, s)
-                           : dispatch_k<64, false>(map, p, bits, counts, idx, zero, status, s);
-    return with_counts ? dispatch_k<128, true>(map, p, bits, counts, idx, zero, status, s)
-                       : dispatch_k<128, false>(map, p, bits, counts, idx, zero, status, s);
+    if (p.E == 32) return dispatch_mode<32>(map, p, bits, counts, idx, cooc, zero, status, s);
+    if (p.E == 64) return dispatch_mode<64>(map, p, bits, counts, idx, cooc, zero, status, s);
+    return dispatch_mode<128>(map, p, bits, counts, idx, cooc, zero, status, s);
 }
 
 }  // namespace dol

@@ -205,7 +205,7 @@ def forward_backward_host(h_logits: torch.Tensor, k, gate=GATE_SIGMOID_NORM, gra
         raise ValueError("h_logits must be a contiguous CPU float32 tensor")
     L, T, E = z.shape
     if device_buffer is None:
-        device_buffer = torch.empty(host_buffer_size(T, E, k, L), dtype=torch.uint8, device="cuda")
+        device_buffer = torch.zeros(host_buffer_size(T, E, k, L), dtype=torch.uint8, device="cuda")
     if h_loss is None:
         h_loss = torch.empty(L, dtype=torch.float32)
     _check("do_forward_backward_host", lib().do_forward_backward_host(
