@@ -250,6 +250,14 @@ def run_ours(args, rank, world, local):
         dl.forward_backward(z, k, w.gate, 1.0, out=out)
 
     warm = max(3, args.warmup)
+    if args.quick:
+        # profiling mode: a few plain steps, nothing else (used under ncu)
+        for i in range(warm + args.steps):
+            step(i)
+        torch.cuda.synchronize()
+        st = dl.device_status(sets[0][1].workspace)
+        print(json.dumps({"quick": True, "steps": warm + args.steps, "status": st}), flush=True)
+        return
     sampler = ClockSampler(local)
     sampler.start()
     for i in range(warm):
@@ -367,6 +375,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--quick", action="store_true",
+                    help="run warmup+steps plain steps and exit (for profilers)")
     args = ap.parse_args()
     if args.impl == "reference":
         rank = int(os.environ.get("RANK", "0"))

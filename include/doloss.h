@@ -103,7 +103,11 @@ do_status do_loss_fwd_bwd(const float *logits, const uint32_t *bits, const int32
                           void *stream);
 
 /* Steps 1-3 in one call on a local window (d_scale = 1): logits in; bits,
- * counts, D, loss, origin_do (may be NULL) and dlogits (may be NULL) out. */
+ * counts, D, loss, origin_do (may be NULL) and dlogits (may be NULL) out.
+ * With the environment variable DOLOSS_LOSS_KERNEL=tcgen05, E = 128, the
+ * sigmoid-normalised gate, k in {1, 2, 4, 8} and dlogits given, the gradient
+ * pass computes W = F D' on the tensor cores instead of gathering rows of D;
+ * the results agree within the tolerances of the ALU kernel. */
 do_status do_forward_backward(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
                               int32_t gate, float grad_scale, uint32_t *bits, int32_t *counts,
                               int32_t *D, float *loss, int64_t *origin_do, float *dlogits,

@@ -4,6 +4,8 @@
 
 #include <climits>
 #include <cstdint>
+#include <cstdlib>
+#include <cstring>
 
 #include "dol_internal.cuh"
 #include "doloss.h"
@@ -24,6 +26,14 @@ do_status check_sizes(int64_t T, int32_t E, int32_t k, int32_t L, Problem *p) {
     p->L = L;
     p->W = (T + 31) / 32;
     return DO_OK;
+}
+
+// The tensor-core loss kernel (one-hot selections times D on tcgen05) runs
+// only when DOLOSS_LOSS_KERNEL=tcgen05 is set: at E = 128 its epilogue costs
+// more than the shared-memory gather of D rows in the ALU kernel.
+bool tcgen05_loss_requested() {
+    const char *v = std::getenv("DOLOSS_LOSS_KERNEL");
+    return v && std::strcmp(v, "tcgen05") == 0;
 }
 
 do_status from_cuda(cudaError_t e) { return e == cudaSuccess ? DO_OK : DO_ERR_CUDA; }
@@ -151,10 +161,19 @@ do_status do_forward_backward(const float *logits, int64_t T, int32_t E, int32_t
         if (e == cudaSuccess)
             e = dol::launch_cooc_reduce(parts, dol::sig_fast_ctas_per_problem(p), n_acc, p, D,
                                         counts, s);
-        if (e == cudaSuccess)
-            e = dol::launch_loss_fast(logits, idx, D, counts, n_acc, p, gate, 1.0f, grad_scale,
-                                      loss, reinterpret_cast<long long *>(origin_do), dlogits,
-                                      reinterpret_cast<double *>(ws + w.partials), done, status, s);
+        if (e == cudaSuccess) {
+            // here D <= T: the two-piece fp16 split of the tensor-core path is exact
+            if (tcgen05_loss_requested() && dol::loss_mma_supported(p, gate, logits, D, dlogits))
+                e = dol::launch_loss_mma(logits, idx, D, counts, n_acc, p, 1.0f, grad_scale, loss,
+                                         reinterpret_cast<long long *>(origin_do), dlogits,
+                                         reinterpret_cast<double *>(ws + w.partials), done, status,
+                                         s);
+            else
+                e = dol::launch_loss_fast(logits, idx, D, counts, n_acc, p, gate, 1.0f, grad_scale,
+                                          loss, reinterpret_cast<long long *>(origin_do), dlogits,
+                                          reinterpret_cast<double *>(ws + w.partials), done,
+                                          status, s);
+        }
         return from_cuda(e);
     }
     cudaError_t e = dol::launch_signatures(logits, p, bits, counts, s);

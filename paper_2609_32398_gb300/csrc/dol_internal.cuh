@@ -76,6 +76,14 @@ cudaError_t launch_idx_from_bits(const uint32_t *bits, const Problem &p, uint8_t
 // counts: when given, R_i = (E - 2k) n_i + T k (D local to these tokens) and
 // n_zero ([L][E], may be null) is cleared once D is read; otherwise R_i is a
 // column sum of D.
+// Tensor-core loss path (E = 128, sigmoid-norm gate, k in {1,2,4,8}, T <= 2^22).
+bool loss_mma_supported(const Problem &p, int gate, const float *logits, const int *D,
+                        const float *dlogits);
+int loss_mma_ctas_per_problem(const Problem &p);
+cudaError_t launch_loss_mma(const float *logits, const uint8_t *idx, const int *D, const int *counts,
+                            int *n_zero, const Problem &p, float d_scale, float grad_scale,
+                            float *loss, long long *origin_do, float *dlogits, double *partials,
+                            int *done, int *status, cudaStream_t s);
 cudaError_t launch_loss_fast(const float *logits, const uint8_t *idx, const int *D,
                              const int *counts, int *n_zero, const Problem &p, int gate,
                              float d_scale, float grad_scale, float *loss, long long *origin_do,
@@ -105,15 +113,17 @@ __device__ __forceinline__ float warp_sum(float v) {
     return v;
 }
 
-// Sum of x[0..n) in a fixed order by a block of nthreads (a power of two):
+// Sum of x[0..n) in a fixed order by the first nthreads (a power of two) of a block:
 // thread i adds x[i], x[i + nthreads], ... in turn, then a fixed tree joins
 // the thread sums.  The result (valid in thread 0) does not depend on timing.
 // red must hold nthreads doubles.  Called by every thread of the block.
 __device__ __forceinline__ double block_sum_fixed(const double *x, int64_t n, double *red,
                                                   int nthreads) {
     double s = 0.0;
-    for (int64_t i = threadIdx.x; i < n; i += nthreads) s += __ldcg(x + i);
-    red[threadIdx.x] = s;
+    if ((int)threadIdx.x < nthreads) {
+        for (int64_t i = threadIdx.x; i < n; i += nthreads) s += __ldcg(x + i);
+        red[threadIdx.x] = s;
+    }
     __syncthreads();
     for (int o = nthreads / 2; o > 0; o >>= 1) {
         if ((int)threadIdx.x < o) red[threadIdx.x] += red[threadIdx.x + o];

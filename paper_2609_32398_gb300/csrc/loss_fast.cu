@@ -35,9 +35,22 @@ namespace {
 constexpr int kLossFastThreads = 256;
 constexpr int kLossFastWarps = kLossFastThreads / 32;
 
+__device__ __forceinline__ float ex2_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__device__ __forceinline__ float rcp_approx(float x) {
+    float y;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// sigmoid(z) = 1 / (1 + 2^(-z log2 e)); for z -> -inf the power is +inf and
+// the reciprocal 0, for z -> +inf the power is 0 and the result 1.
 __device__ __forceinline__ float sigmoid_fast(float z) {
-    const float e = __expf(-fmaxf(z, -80.0f));
-    return __fdividef(1.0f, 1.0f + e);
+    return rcp_approx(1.0f + ex2_approx(z * -1.4426950408889634f));
 }
 
 template <int K>
@@ -82,7 +95,7 @@ struct LossArgs {
 };
 
 template <int E, int K, int kGate, bool kRFromCounts>
-__global__ void __launch_bounds__(kLossFastThreads)
+__global__ void __launch_bounds__(kLossFastThreads, 3)
 loss_fast_kernel(const LossArgs a) {
     constexpr int G = E / 16;    // lanes per token
     constexpr int TPW = 32 / G;  // tokens per warp pass
@@ -224,9 +237,10 @@ loss_fast_kernel(const LossArgs a) {
             for (int e = 1; e < 16; ++e) mx = fmaxf(mx, zz[e]);
 #pragma unroll
             for (int o = G / 2; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, o));
+            const float mxs = mx * 1.4426950408889634f;
 #pragma unroll
             for (int e = 0; e < 16; ++e) {
-                gv[e] = __expf(zz[e] - mx);
+                gv[e] = ex2_approx(fmaf(zz[e], 1.4426950408889634f, -mxs));
                 den += gv[e];
                 num = fmaf(gv[e], w[e], num);
             }
@@ -240,7 +254,9 @@ loss_fast_kernel(const LossArgs a) {
         const float A = num * inv;
         if (valid && g == 0) tok_sum += (double)A;
         if (dzl && valid) {
+            // dz = c/S * jac * (w - A) = jac * (cs w - cs A)
             const float cs = a.coef * inv;
+            const float csA = cs * A;
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 float4 o;
@@ -248,8 +264,8 @@ loss_fast_kernel(const LossArgs a) {
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
                     const float s = gv[4 * c + e];
-                    const float jac = (kGate == 0) ? s - s * s : s;
-                    op[e] = cs * jac * (w[4 * c + e] - A);
+                    const float jac = (kGate == 0) ? fmaf(-s, s, s) : s;
+                    op[e] = jac * fmaf(cs, w[4 * c + e], -csA);
                 }
                 *reinterpret_cast<float4 *>(dzl + t * E + c * Q + 4 * g) = o;
             }
@@ -423,7 +439,7 @@ void loss_fast_grid(const Problem &p, int *P, int *tokens_per_cta) {
     int dev = 0, sms = 148;
     if (cudaGetDevice(&dev) == cudaSuccess)
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    int64_t want = (int64_t)sms * 2 / p.L;  // two CTAs fit on an SM: one wave
+    int64_t want = (int64_t)sms * 3 / p.L;  // three CTAs fit on an SM: one wave
     if (want < 1) want = 1;
     int64_t tpc = (p.T + want - 1) / want;
     tpc = (tpc + 31) / 32 * 32;

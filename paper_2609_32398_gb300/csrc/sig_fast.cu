@@ -255,14 +255,25 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W,
 
         if (idx && valid) store_idx<K>(idx + (layer * T + t) * K, sel);
         if (kCooc && valid) {
-            // c_ab += 1 for every pair a <= b of selected experts (a = b gives n_a)
+            // c_ab += 1 for every pair a < b of selected experts (the counts on
+            // the diagonal come from the signature words below)
+            int so[K];
 #pragma unroll
-            for (int q1 = 0; q1 < K; ++q1)
+            for (int q = 0; q < K; ++q) so[q] = sel[q];
 #pragma unroll
-                for (int q2 = q1; q2 < K; ++q2) {
-                    const int a = min(sel[q1], sel[q2]), b = max(sel[q1], sel[q2]);
-                    atomicAdd(&s_cooc[s_rowoff[a] + b], 1u);
+            for (int i = 1; i < K; ++i)  // insertion sort of K indices (static network)
+#pragma unroll
+                for (int j = i; j > 0; --j) {
+                    const int lo = min(so[j - 1], so[j]), hi = max(so[j - 1], so[j]);
+                    so[j - 1] = lo;
+                    so[j] = hi;
                 }
+#pragma unroll
+            for (int q1 = 0; q1 < K - 1; ++q1) {
+                uint32_t *row = s_cooc + s_rowoff[so[q1]];
+#pragma unroll
+                for (int q2 = q1 + 1; q2 < K; ++q2) atomicAdd(row + so[q2], 1u);
+            }
         }
         uint32_t m[R];
 #pragma unroll
@@ -278,13 +289,18 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W,
         for (int r = 0; r < R; ++r) {
             const uint32_t word = transpose32(valid ? m[r] : 0u, lane);
             bits[(layer * E + 32 * r + lane) * W + w] = word;
-            if (kCounts) cnt[r] += __popc(word);
+            if (kCounts || kCooc) cnt[r] += __popc(word);
         }
     }
     if (kCounts) {
 #pragma unroll
         for (int r = 0; r < R; ++r)
             if (cnt[r]) atomicAdd(&counts[layer * E + 32 * r + lane], (int)cnt[r]);
+    }
+    if (kCooc) {  // counts n_a on the triangle's diagonal
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+            if (cnt[r]) atomicAdd(&s_cooc[s_rowoff[32 * r + lane] + 32 * r + lane], cnt[r]);
     }
     if (kCooc) {
         // all consumer warps have counted: store this CTA's triangle for the

@@ -240,3 +240,21 @@ def test_repeated_calls_reuse_workspace(dl):
             first = cur
         assert all(torch.equal(a, b) for a, b in zip(first, cur))
     assert dl.device_status(out.workspace) == 0
+
+
+@pytest.mark.parametrize("T,k,L", [(65536, 8, 1), (4096 + 33, 4, 2), (300, 1, 1), (1000, 2, 3)])
+def test_tcgen05_loss_kernel(dl, monkeypatch, T, k, L):
+    """The tensor-core gradient pass, chosen by DOLOSS_LOSS_KERNEL=tcgen05."""
+    z = workloads.random_logits(T, 128, L=L, seed=T + k, ties=T < 2000)
+    monkeypatch.setenv("DOLOSS_LOSS_KERNEL", "tcgen05")
+    out = gpu_run(dl, z, k, workloads.GATE_SIGMOID_NORM, grad_scale=2.0)
+    monkeypatch.delenv("DOLOSS_LOSS_KERNEL")
+    ref = gpu_run(dl, z, k, workloads.GATE_SIGMOID_NORM, grad_scale=2.0)
+    for name in ("bits", "counts", "D", "origin_do"):
+        assert torch.equal(getattr(out, name), getattr(ref, name)), name
+    for l in range(L):
+        if T <= 8192:
+            assert_layer(out, l, z[l].numpy(), k, workloads.GATE_SIGMOID_NORM, grad_scale=2.0)
+        assert float(out.loss[l]) == pytest.approx(float(ref.loss[l]), rel=1e-5)
+        err = (out.dlogits[l] - ref.dlogits[l]).abs().max() / ref.dlogits[l].abs().max()
+        assert float(err) <= 1e-5
