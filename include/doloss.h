@@ -138,6 +138,34 @@ do_status do_forward_backward_host(const float *h_logits, int64_t T, int32_t E, 
 
 size_t do_host_buffer_size(int64_t T, int32_t E, int32_t k, int32_t L);
 
+/* Largest workspace, in bytes, that do_forward_backward_static can hold. */
+#define DO_STATIC_SCRATCH_BYTES ((size_t)16 << 20)
+
+/* do_forward_backward for callers that cannot allocate device memory (an
+ * embedding C host without a device allocator, or a process that has handed
+ * its spare HBM to its own pool).  The paper has no counterpart: it is an
+ * interface variant of steps 1-3, with the same arguments and results as
+ * do_forward_backward except that the workspace is a fixed 16 MiB array
+ * inside the library, one per device.
+ *  - Sizes whose do_workspace_size exceeds DO_STATIC_SCRATCH_BYTES are
+ *    rejected with DO_ERR_WORKSPACE before anything is launched (for
+ *    E = 128, k = 8, L = 1 that is T above 984,896 tokens).
+ *  - Unlike the other entry points it keeps state: the first call on a device
+ *    (with that device current) looks up the array's address, zero-fills the
+ *    array and synchronizes the device; make that first call before any
+ *    stream capture begins.  Every call then clears the parts that must start
+ *    at zero with cudaMemsetAsync on `stream`.
+ *  - status_flags (device int32, may be NULL) receives the device status
+ *    word of this call, copied on `stream`: bit 0 = a Hamming row sum did
+ *    not fit int32, bit 1 = a bounded device wait ran out.
+ *  - All calls share one array per device: calls that overlap in time (on
+ *    two streams or from two threads) race.  Serialize them on one stream.
+ *  - Allocates nothing (no cudaMalloc, no allocating library). */
+do_status do_forward_backward_static(const float *logits, int64_t T, int32_t E, int32_t k,
+                                     int32_t L, int32_t gate, float grad_scale, uint32_t *bits,
+                                     int32_t *counts, int32_t *D, float *loss, int64_t *origin_do,
+                                     float *dlogits, int32_t *status_flags, void *stream);
+
 /* A static description of a status code. */
 const char *do_status_string(int32_t status);
 

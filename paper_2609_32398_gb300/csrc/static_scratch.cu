@@ -1,0 +1,95 @@
+// do_forward_backward_static (declared in include/doloss.h): the fused path
+// of do_forward_backward with its workspace taken from a fixed device array
+// inside libdoloss instead of from the caller.
+//
+// It serves callers that cannot allocate device memory at call time: a plain C
+// host that embeds the library without any device allocator of its own, or a
+// serving process that hands all spare HBM to its own pool at start-up and
+// forbids cudaMalloc afterwards (an allocation there would fail or fragment
+// the pool).  Nothing here calls cudaMalloc, cudaFree or an allocating library.
+//
+// The scratch is one array per device (one per CUDA context), so calls that
+// overlap in time — on two streams, or from two host threads — share it and
+// race; such callers must serialize their calls on one stream.
+#include <cuda_runtime.h>
+
+#include <mutex>
+
+#include "dol_internal.cuh"
+#include "doloss.h"
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+
+static __device__ __align__(256) unsigned char g_scratch[DO_STATIC_SCRATCH_BYTES];
+
+std::mutex g_mu;
+void *g_scratch_ptr[kMaxDevices] = {};
+
+// Address of the scratch on the current device.  The first call on a device
+// looks it up (the device must be current, as it is here) and zero-fills it,
+// then waits for the device so that the fill is complete before any stream
+// uses the array.
+do_status scratch_on_current_device(void **out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return DO_ERR_CUDA;
+    if (dev < 0 || dev >= kMaxDevices) return DO_ERR_UNSUPPORTED;
+    std::lock_guard<std::mutex> lock(g_mu);
+    if (!g_scratch_ptr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_scratch) != cudaSuccess || !p) return DO_ERR_CUDA;
+        if (cudaMemset(p, 0, DO_STATIC_SCRATCH_BYTES) != cudaSuccess) return DO_ERR_CUDA;
+        if (cudaDeviceSynchronize() != cudaSuccess) return DO_ERR_CUDA;
+        g_scratch_ptr[dev] = p;
+    }
+    *out = g_scratch_ptr[dev];
+    return DO_OK;
+}
+
+}  // namespace
+
+extern "C" do_status do_forward_backward_static(const float *logits, int64_t T, int32_t E,
+                                                int32_t k, int32_t L, int32_t gate,
+                                                float grad_scale, uint32_t *bits, int32_t *counts,
+                                                int32_t *D, float *loss, int64_t *origin_do,
+                                                float *dlogits, int32_t *status_flags,
+                                                void *stream) {
+    // the sizes are checked by do_workspace_size (0 = invalid) before anything else
+    const size_t need = do_workspace_size(T, E, k, L);
+    if (need == 0) {
+        if (T < 1 || E < 1 || k < 1 || k > E || L < 1) return DO_ERR_INVALID_ARG;
+        return DO_ERR_UNSUPPORTED;
+    }
+    if (need > DO_STATIC_SCRATCH_BYTES) return DO_ERR_WORKSPACE;
+    if (!logits || !bits || !counts || !D || !loss) return DO_ERR_INVALID_ARG;
+    if (status_flags && reinterpret_cast<uintptr_t>(status_flags) % 4 != 0)
+        return DO_ERR_INVALID_ARG;
+    void *ws = nullptr;
+    do_status st = scratch_on_current_device(&ws);
+    if (st != DO_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    // What must be zero when a call starts: the status word and the done
+    // counters (the first 256-byte-aligned span) and the counts accumulator
+    // (the last span).  The kernels leave them zero after a complete call;
+    // clearing them here also recovers from a call that gave up on a wait.
+    dol::Problem p;
+    p.T = T;
+    p.E = E;
+    p.k = k;
+    p.L = L;
+    p.W = (T + 31) / 32;
+    const dol::WsLayout w = dol::ws_layout(p);
+    char *base = static_cast<char *>(ws);
+    if (cudaMemsetAsync(base, 0, w.partials, s) != cudaSuccess) return DO_ERR_CUDA;
+    if (w.total > w.n_acc && cudaMemsetAsync(base + w.n_acc, 0, w.total - w.n_acc, s) != cudaSuccess)
+        return DO_ERR_CUDA;
+    st = do_forward_backward(logits, T, E, k, L, gate, grad_scale, bits, counts, D, loss, origin_do,
+                             dlogits, ws, DO_STATIC_SCRATCH_BYTES, stream);
+    if (st != DO_OK) return st;
+    if (status_flags &&
+        cudaMemcpyAsync(status_flags, base, sizeof(int32_t), cudaMemcpyDeviceToDevice, s) !=
+            cudaSuccess)
+        return DO_ERR_CUDA;
+    return DO_OK;
+}

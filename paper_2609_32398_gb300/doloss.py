@@ -35,6 +35,8 @@ EXPORTS = {
                                   "p", "p", "sz", "p"], "i32"),
     "do_host_buffer_size": (["i64", "i32", "i32", "i32"], "sz"),
     "do_status_string": (["i32"], "str"),
+    "do_forward_backward_static": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p", "p",
+                                    "p", "p", "p", "p", "p"], "i32"),
 }
 
 _CT = {"p": ctypes.c_void_p, "i64": ctypes.c_int64, "i32": ctypes.c_int32,
@@ -213,3 +215,19 @@ def forward_backward_host(h_logits: torch.Tensor, k, gate=GATE_SIGMOID_NORM, gra
         _ptr(h_counts), _ptr(h_D), device_buffer.data_ptr(), device_buffer.numel(),
         torch.cuda.current_stream(device_buffer.device).cuda_stream))
     return h_loss
+
+
+def forward_backward_static(logits, k, out: Buffers, gate=GATE_SIGMOID_NORM, grad_scale=1.0,
+                            status_flags: torch.Tensor | None = None):
+    """do_forward_backward_static: steps 1-3 with the library's own fixed
+    scratch array; out.workspace is not used.  status_flags: int32 [1] on the
+    device, or None."""
+    z = _as3d(logits)
+    L, T, E = z.shape
+    if out.shape != (L, T, E, k):
+        raise ValueError("output buffers were made for another shape")
+    _check("do_forward_backward_static", lib().do_forward_backward_static(
+        z.data_ptr(), T, E, k, L, gate, grad_scale, out.bits.data_ptr(), out.counts.data_ptr(),
+        out.D.data_ptr(), out.loss.data_ptr(), out.origin_do.data_ptr(), _ptr(out.dlogits),
+        _ptr(status_flags), _stream(z)))
+    return out

@@ -1,0 +1,53 @@
+"""do_forward_backward_static: the fused path with the library's fixed scratch
+array gives the results of do_forward_backward, call after call, and rejects
+sizes whose workspace exceeds the array before launching anything."""
+import ctypes
+
+import pytest
+import torch
+
+from paper_2609_32398_gb300 import workloads
+
+pytestmark = pytest.mark.gpu
+
+LOSS_RTOL = 1e-5
+GRAD_TOL = 1e-5
+
+
+@pytest.fixture(scope="module")
+def dl():
+    import paper_2609_32398_gb300.doloss as m
+
+    m.lib()
+    return m
+
+
+@pytest.mark.parametrize("T,E,k,L,gate", [(8192 + 17, 128, 8, 1, 0), (3000, 96, 3, 2, 1),
+                                          (65536, 128, 8, 1, 0)])
+def test_static_scratch_matches_workspace_path(dl, T, E, k, L, gate):
+    z = workloads.random_logits(T, E, L=L, seed=T + E).cuda()
+    ref = dl.forward_backward(z, k, gate, grad_scale=1.5)
+    assert dl.device_status(ref.workspace) == 0
+    flags = torch.full((1,), -1, dtype=torch.int32, device="cuda")
+    for _ in range(2):  # two consecutive calls on the same scratch
+        out = dl.Buffers(L, T, E, k, "cuda")
+        dl.forward_backward_static(z, k, out, gate, grad_scale=1.5, status_flags=flags)
+        torch.cuda.synchronize()
+        assert int(flags[0]) == 0
+        for name in ("bits", "counts", "D", "origin_do"):
+            assert torch.equal(getattr(out, name), getattr(ref, name)), name
+        for l in range(L):
+            assert float(out.loss[l]) == pytest.approx(float(ref.loss[l]), rel=LOSS_RTOL)
+            err = (out.dlogits[l] - ref.dlogits[l]).abs().max() / ref.dlogits[l].abs().max()
+            assert float(err) <= GRAD_TOL
+
+
+def test_static_scratch_rejects_oversized_problems(dl):
+    T, E, k = 984896 + 32, 128, 8
+    assert dl.workspace_size(T, E, k, 1) > (16 << 20)
+    small = torch.zeros(64, device="cuda")
+    p = ctypes.c_void_p(small.data_ptr())   # never dereferenced: the size check fails first
+    st = dl.lib().do_forward_backward_static(p, T, E, k, 1, 0, 1.0, p, p, p, p, None, None, None,
+                                             None)
+    assert st == 6, dl.status_string(st)    # DO_ERR_WORKSPACE
+    assert dl.workspace_size(984896, E, k, 1) <= (16 << 20)
