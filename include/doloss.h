@@ -104,10 +104,11 @@ do_status do_loss_fwd_bwd(const float *logits, const uint32_t *bits, const int32
 
 /* Steps 1-3 in one call on a local window (d_scale = 1): logits in; bits,
  * counts, D, loss, origin_do (may be NULL) and dlogits (may be NULL) out.
- * With the environment variable DOLOSS_LOSS_KERNEL=tcgen05, E = 128, the
- * sigmoid-normalised gate, k in {1, 2, 4, 8} and dlogits given, the gradient
- * pass computes W = F D' on the tensor cores instead of gathering rows of D;
- * the results agree within the tolerances of the ALU kernel. */
+ * With E = 128, the sigmoid-normalised gate, k in {1, 2, 4, 8}, T <= 66052
+ * and dlogits given, the gradient pass computes V = F D' on the tensor cores
+ * (F the one-hot selections, D' = D with -R on the diagonal); elsewhere, or
+ * with the environment variable DOLOSS_LOSS_KERNEL=alu, it gathers rows of D'
+ * on the ALU.  The two agree within the stated tolerances. */
 do_status do_forward_backward(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
                               int32_t gate, float grad_scale, uint32_t *bits, int32_t *counts,
                               int32_t *D, float *loss, int64_t *origin_do, float *dlogits,
@@ -149,7 +150,7 @@ size_t do_host_buffer_size(int64_t T, int32_t E, int32_t k, int32_t L);
  * inside the library, one per device.
  *  - Sizes whose do_workspace_size exceeds DO_STATIC_SCRATCH_BYTES are
  *    rejected with DO_ERR_WORKSPACE before anything is launched (for
- *    E = 128, k = 8, L = 1 that is T above 984,896 tokens).
+ *    E = 128, k = 8, L = 1 that is T above about 0.97 million tokens).
  *  - Unlike the other entry points it keeps state: the first call on a device
  *    (with that device current) looks up the array's address, zero-fills the
  *    array and synchronizes the device; make that first call before any

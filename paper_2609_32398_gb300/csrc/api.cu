@@ -28,12 +28,12 @@ do_status check_sizes(int64_t T, int32_t E, int32_t k, int32_t L, Problem *p) {
     return DO_OK;
 }
 
-// The tensor-core loss kernel (one-hot selections times D on tcgen05) runs
-// only when DOLOSS_LOSS_KERNEL=tcgen05 is set: at E = 128 its epilogue costs
-// more than the shared-memory gather of D rows in the ALU kernel.
-bool tcgen05_loss_requested() {
+// The fused path takes the tensor-core loss kernel (one-hot selections times
+// D' on tcgen05) wherever it applies; DOLOSS_LOSS_KERNEL=alu selects the ALU
+// kernel (a shared-memory gather of D rows) instead.
+bool alu_loss_requested() {
     const char *v = std::getenv("DOLOSS_LOSS_KERNEL");
-    return v && std::strcmp(v, "tcgen05") == 0;
+    return v && std::strcmp(v, "alu") == 0;
 }
 
 do_status from_cuda(cudaError_t e) { return e == cudaSuccess ? DO_OK : DO_ERR_CUDA; }
@@ -154,23 +154,28 @@ do_status do_forward_backward(const float *logits, int64_t T, int32_t E, int32_t
         uint8_t *idx = reinterpret_cast<uint8_t *>(ws + w.idx);
         uint32_t *parts = reinterpret_cast<uint32_t *>(ws + w.cooc_parts);
         int *n_acc = reinterpret_cast<int *>(ws + w.n_acc);
-        const dol::ZeroSpans zero = {{done, nullptr, nullptr}, {(int64_t)p.L, 0, 0}};
+        // origin_do is summed by the reduction kernel (integer atomics): zero it first
+        const dol::ZeroSpans zero = {{done, reinterpret_cast<int *>(origin_do), nullptr},
+                                     {(int64_t)p.L, origin_do ? 2 * (int64_t)p.L : 0, 0}};
         int *status = reinterpret_cast<int *>(ws);
+        // D <= T here (one window of tokens): the two-piece fp16 split of the
+        // tensor-core path is exact when R < 2^23 (checked by loss_mma_supported)
+        const bool mma = !alu_loss_requested() &&
+                         dol::loss_mma_supported(p, gate, logits, D, dlogits);
+        unsigned char *bimg = mma ? reinterpret_cast<unsigned char *>(ws + w.bimg) : nullptr;
         cudaError_t e =
             dol::launch_signatures_fast(logits, p, bits, n_acc, idx, parts, zero, status, s);
         if (e == cudaSuccess)
             e = dol::launch_cooc_reduce(parts, dol::sig_fast_ctas_per_problem(p), n_acc, p, D,
-                                        counts, s);
+                                        counts, bimg, reinterpret_cast<long long *>(origin_do), s);
         if (e == cudaSuccess) {
-            // here D <= T: the two-piece fp16 split of the tensor-core path is exact
-            if (tcgen05_loss_requested() && dol::loss_mma_supported(p, gate, logits, D, dlogits))
-                e = dol::launch_loss_mma(logits, idx, D, counts, n_acc, p, 1.0f, grad_scale, loss,
-                                         reinterpret_cast<long long *>(origin_do), dlogits,
+            if (mma)
+                e = dol::launch_loss_mma(logits, idx, bimg, n_acc, p, 1.0f, grad_scale, loss, dlogits,
                                          reinterpret_cast<double *>(ws + w.partials), done, status,
                                          s);
             else
                 e = dol::launch_loss_fast(logits, idx, D, counts, n_acc, p, gate, 1.0f, grad_scale,
-                                          loss, reinterpret_cast<long long *>(origin_do), dlogits,
+                                          loss, nullptr, dlogits,
                                           reinterpret_cast<double *>(ws + w.partials), done,
                                           status, s);
         }

@@ -1,12 +1,16 @@
 // Reduction of the per-CTA co-occurrence triangles of the fused path.
 //   c_ab = sum_t f_at f_bt, c_aa = n_a, and the Hamming distance
 //   D_ab = n_a + n_b - 2 c_ab                                   (App. C.3)
+// and, alongside, Eq. origin_do: sum over a != b of D_ab^2 (exact integer
+// adds, one per CTA).
 // The counts n_a were already summed (one atomic per expert and CTA) by the
 // signatures kernel.  A CTA owns 32 consecutive triangle words; its 32 warps
 // each sum a strided subset of the partials with independent loads, and the
 // 32 warp sums are added in a fixed order, so D is an exact integer result
 // independent of scheduling.  The kernel writes both halves of the symmetric
 // D and the counts.
+#include <cuda_fp16.h>
+
 #include "dol_internal.cuh"
 #include "tma.cuh"
 
@@ -16,10 +20,18 @@ namespace {
 constexpr int kRedWarps = 32;
 constexpr int kRedThreads = kRedWarps * 32;
 
+__device__ __forceinline__ void put_pieces(unsigned char *img, int n, int k, bool diag, int v) {
+    int h, l;
+    dprime_pieces(diag, v, &h, &l);
+    *reinterpret_cast<__half *>(img + sw128_k16_offset(n, k, 256)) = __int2half_rn(h);
+    *reinterpret_cast<__half *>(img + sw128_k16_offset(128 + n, k, 256)) = __int2half_rn(l);
+}
+
 template <int E>
 __global__ void __launch_bounds__(kRedThreads)
 cooc_reduce_kernel(const uint32_t *__restrict__ partials, int P1, const int *__restrict__ n_acc,
-                   int *__restrict__ D, int *__restrict__ counts) {
+                   int *__restrict__ D, int *__restrict__ counts, unsigned char *__restrict__ bimg,
+                   long long *__restrict__ origin_do, long long r_base, int r_mult) {
     constexpr int kWords = cooc_row_offset<E>(E);
     __shared__ uint32_t s_sum[kRedWarps][33];
     const int e = threadIdx.x & 31, wp = threadIdx.x >> 5;
@@ -40,35 +52,53 @@ cooc_reduce_kernel(const uint32_t *__restrict__ partials, int P1, const int *__r
     }
     s_sum[wp][e] = acc[0] + acc[1] + acc[2] + acc[3];
     __syncthreads();
-    if (wp != 0 || word >= kWords) return;
-    uint32_t c = 0;
+    if (wp != 0) return;
+    long long sq = 0;  // this word's part of sum_{a != b} D_ab^2
+    if (word < kWords) {
+        uint32_t c = 0;
 #pragma unroll
-    for (int q = 0; q < kRedWarps; ++q) c += s_sum[q][e];
-    // word -> (a, b): the row whose offset range holds it
-    int lo = 0, hi = E - 1;
-    while (lo < hi) {
-        const int mid = (lo + hi + 1) >> 1;
-        if (cooc_row_offset<E>(mid) <= word) lo = mid;
-        else hi = mid - 1;
+        for (int q = 0; q < kRedWarps; ++q) c += s_sum[q][e];
+        // word -> (a, b): the row whose offset range holds it
+        int lo = 0, hi = E - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (cooc_row_offset<E>(mid) <= word) lo = mid;
+            else hi = mid - 1;
+        }
+        const int a = lo;
+        const int b = (a & ~3) + (word - cooc_row_offset<E>(a));
+        const int *nl = n_acc + (size_t)layer * E;
+        int *Dl = D + (size_t)layer * E * E;
+        unsigned char *img = (E == 128 && bimg) ? bimg + (size_t)layer * kBImageBytes : nullptr;
+        if (b < a) {
+            // alignment padding of row a: nothing to write
+        } else if (a == b) {
+            Dl[a * E + a] = 0;
+            counts[(size_t)layer * E + a] = (int)c;
+            // R_a = (E - 2k) n_a + T k (every row of the co-occurrence sums to k n_a)
+            if (img) put_pieces(img, a, a, true, (int)(r_base + (long long)r_mult * (long long)c));
+        } else {
+            const int d = nl[a] + nl[b] - 2 * (int)c;
+            Dl[a * E + b] = d;
+            Dl[b * E + a] = d;
+            if (img) {
+                put_pieces(img, a, b, false, d);
+                put_pieces(img, b, a, false, d);
+            }
+            sq = 2 * (long long)d * (long long)d;
+        }
     }
-    const int a = lo;
-    const int b = (a & ~3) + (word - cooc_row_offset<E>(a));
-    if (b < a) return;  // alignment padding of row a
-    const int *nl = n_acc + (size_t)layer * E;
-    int *Dl = D + (size_t)layer * E * E;
-    if (a == b) {
-        Dl[a * E + a] = 0;
-        counts[(size_t)layer * E + a] = (int)c;
-    } else {
-        const int d = nl[a] + nl[b] - 2 * (int)c;
-        Dl[a * E + b] = d;
-        Dl[b * E + a] = d;
+    if (origin_do) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(kFull, sq, o);
+        if (e == 0 && sq)
+            atomicAdd(reinterpret_cast<unsigned long long *>(origin_do + layer), (unsigned long long)sq);
     }
 }
 
 template <int E>
 cudaError_t run_reduce(const uint32_t *partials, int P1, const int *n_acc, const Problem &p, int *D,
-                       int *counts, cudaStream_t s) {
+                       int *counts, unsigned char *bimg, long long *origin_do, cudaStream_t s) {
     constexpr int kWords = cooc_row_offset<E>(E);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((kWords + 31) / 32, (unsigned)p.L);
@@ -79,16 +109,20 @@ cudaError_t run_reduce(const uint32_t *partials, int P1, const int *n_acc, const
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, cooc_reduce_kernel<E>, partials, P1, n_acc, D, counts);
+    const long long r_base = p.T * (long long)p.k;
+    const int r_mult = E - 2 * p.k;
+    return cudaLaunchKernelEx(&cfg, cooc_reduce_kernel<E>, partials, P1, n_acc, D, counts, bimg,
+                              origin_do, r_base, r_mult);
 }
 
 }  // namespace
 
 cudaError_t launch_cooc_reduce(const uint32_t *partials, int P1, const int *n_acc, const Problem &p,
-                               int *D, int *counts, cudaStream_t s) {
-    if (p.E == 32) return run_reduce<32>(partials, P1, n_acc, p, D, counts, s);
-    if (p.E == 64) return run_reduce<64>(partials, P1, n_acc, p, D, counts, s);
-    if (p.E == 128) return run_reduce<128>(partials, P1, n_acc, p, D, counts, s);
+                               int *D, int *counts, unsigned char *bimg, long long *origin_do,
+                               cudaStream_t s) {
+    if (p.E == 32) return run_reduce<32>(partials, P1, n_acc, p, D, counts, nullptr, origin_do, s);
+    if (p.E == 64) return run_reduce<64>(partials, P1, n_acc, p, D, counts, nullptr, origin_do, s);
+    if (p.E == 128) return run_reduce<128>(partials, P1, n_acc, p, D, counts, bimg, origin_do, s);
     return cudaErrorInvalidValue;
 }
 

@@ -40,8 +40,9 @@ struct ZeroSpans {
 //   cooc_parts      [L][P1][triangle words] uint32, per-CTA co-occurrence counts
 //   n_acc           [L][E] int32, counts summed by the signatures CTAs (kept at
 //                   zero between calls: the loss kernel clears it after use)
+//   bimg            [L][kBImageBytes], the fp16 image of D' (E = 128 only)
 struct WsLayout {
-    size_t done, partials, idx, cooc_parts, n_acc, total;
+    size_t done, partials, idx, cooc_parts, n_acc, bimg, total;
     int max_parts;  // partial slots per problem
 };
 // Signatures CTAs per problem on the fast path: min(SMs, kMaxSigCtas) / L.
@@ -80,10 +81,12 @@ cudaError_t launch_idx_from_bits(const uint32_t *bits, const Problem &p, uint8_t
 bool loss_mma_supported(const Problem &p, int gate, const float *logits, const int *D,
                         const float *dlogits);
 int loss_mma_ctas_per_problem(const Problem &p);
-cudaError_t launch_loss_mma(const float *logits, const uint8_t *idx, const int *D, const int *counts,
+// bimg: the fp16 image of D' written by launch_cooc_reduce for these tokens
+// (which also gives origin_do on this path).
+cudaError_t launch_loss_mma(const float *logits, const uint8_t *idx, const unsigned char *bimg,
                             int *n_zero, const Problem &p, float d_scale, float grad_scale,
-                            float *loss, long long *origin_do, float *dlogits, double *partials,
-                            int *done, int *status, cudaStream_t s);
+                            float *loss, float *dlogits, double *partials, int *done, int *status,
+                            cudaStream_t s);
 cudaError_t launch_loss_fast(const float *logits, const uint8_t *idx, const int *D,
                              const int *counts, int *n_zero, const Problem &p, int gate,
                              float d_scale, float grad_scale, float *loss, long long *origin_do,
@@ -98,10 +101,37 @@ __host__ __device__ constexpr int cooc_row_offset(int a) {
     return a * E - 8 * (a / 4) * (a / 4 - 1) - 4 * (a % 4) * (a / 4);
 }
 
+// The matrix D' of the tensor-core loss kernel (E = 128): D'_ab = D_ab off the
+// diagonal, D'_aa = -R_a, stored as two fp16 pieces D' = 2048 hi + lo, both
+// exact: off the diagonal (0 <= D <= 2^16) hi = D >> 11 and lo = D & 2047; on
+// the diagonal (0 <= R < 2^23) -R = 2048 (-a) + (-b) with a = 2 round(R / 4096)
+// even and |b| <= 2048.  The image is the shared-memory operand B of that
+// kernel: rows n = 0..127 hold hi of column n, rows 128 + n lo, K-major with
+// 128-byte swizzle (two K atoms of 64 columns, 256 rows of 128 bytes each).
+constexpr int kBImageBytes = 2 * 256 * 128;
+__host__ __device__ __forceinline__ uint32_t sw128_k16_offset(int row, int k, int rows) {
+    const int atom = k >> 6, kc = k & 63;
+    return (uint32_t)(atom * rows * 128 + row * 128 + ((((kc >> 3) ^ (row & 7))) << 4) + (kc & 7) * 2);
+}
+__host__ __device__ __forceinline__ void dprime_pieces(bool diag, int v, int *hi, int *lo) {
+    if (diag) {  // v = R
+        const int a2 = 2 * ((v + 2048) >> 12);
+        *hi = -a2;
+        *lo = -(v - 2048 * a2);
+    } else {     // v = D
+        *hi = v >> 11;
+        *lo = v & 2047;
+    }
+}
+
 int sig_fast_ctas_per_problem(const Problem &p);
 size_t cooc_partial_words(int E);
+// bimg ([L][kBImageBytes], E = 128 only, may be null): the fp16 image of D'
+// for the tensor-core loss kernel, written alongside D.  origin_do (may be
+// null) must be zero on entry: sum_{a != b} D_ab^2 is added to it.
 cudaError_t launch_cooc_reduce(const uint32_t *partials, int P1, const int *n_acc, const Problem &p,
-                               int *D, int *counts, cudaStream_t s);
+                               int *D, int *counts, unsigned char *bimg, long long *origin_do,
+                               cudaStream_t s);
 
 // ---------------------------------------------------------------- device helpers
 
@@ -130,6 +160,18 @@ __device__ __forceinline__ double block_sum_fixed(const double *x, int64_t n, do
         __syncthreads();
     }
     return red[0];
+}
+
+// Sum of x[0..n) by one full warp in a fixed order: lane l adds x[l],
+// x[l + 32], ... in turn, then a fixed butterfly joins the lane sums.  The
+// result (in every lane) does not depend on timing.
+__device__ __forceinline__ double warp_sum_fixed(const double *x, int64_t n) {
+    const int lane = threadIdx.x & 31;
+    double s = 0.0;
+    for (int64_t i = lane; i < n; i += 32) s += __ldcg(x + i);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(kFull, s, o);
+    return s;
 }
 
 __device__ __forceinline__ float warp_max(float v) {

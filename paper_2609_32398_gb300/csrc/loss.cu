@@ -247,7 +247,8 @@ WsLayout ws_layout(const Problem &p) {
                                                   cooc_partial_words(p.E)
                                             : 0;
     w.n_acc = up(w.cooc_parts + parts);
-    w.total = up(w.n_acc + ((fast_k && fast_e) ? sizeof(int) * (size_t)p.L * p.E : 0));
+    w.bimg = up(w.n_acc + ((fast_k && fast_e) ? sizeof(int) * (size_t)p.L * p.E : 0));
+    w.total = up(w.bimg + ((fast_k && p.E == 128) ? (size_t)kBImageBytes * (size_t)p.L : 0));
     return w;
 }
 

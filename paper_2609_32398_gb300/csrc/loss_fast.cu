@@ -291,11 +291,9 @@ loss_fast_kernel(const LossArgs a) {
     if (!s_last) return;
     // last CTA of this problem: fixed-order sum of the partials, origin_do
     __threadfence();
-    {
-        __shared__ double s_red[kLossFastThreads];
-        const double sum = block_sum_fixed(a.partials + (int64_t)layer * P, P, s_red,
-                                           kLossFastThreads);
-        if (threadIdx.x == 0) {
+    if (warp == 0) {
+        const double sum = warp_sum_fixed(a.partials + (int64_t)layer * P, P);
+        if (lane == 0) {
             a.loss[layer] = (float)(sum * a.scale);
             a.done[layer] = 0;
         }

@@ -1,28 +1,43 @@
-// Step 3 on the tensor cores (E = 128, sigmoid-norm gate, k in {1, 2, 4, 8}):
-// the surrogate DO-loss and its gradient (Sec. 3.1.3, Eq. do_loss).
+// Step 3 on the tensor cores (E = 128, sigmoid-norm gate, k in {1, 2, 4, 8},
+// D from the co-occurrence counts of the same tokens): the surrogate DO-loss
+// and its gradient (Sec. 3.1.3, Eq. do_loss).
 //
-// With F_t the one-hot rows of the selected experts, G = F D is the k-row
-// gather G_ti = sum_{j in S_t} D_ji, and
-//   w_ti = f_ti R_i - G_ti,   A_t = (sum_{j in S_t} s_j R_j - sum_i s_i G_ti) / S,
-//   dz_ti = c/S s_i (1 - s_i) (w_ti - A_t)
-//         = -c/S jac_i (G_ti + A_t)  +  [i in S_t] c/S jac_i R_i,
-// with s = sigmoid(z), S = sum_i s_i, jac = s (1 - s), c = grad_scale d_scale/(m^2 k).
-// G is computed exactly on the tensor cores: F is 0/1 in fp16 and D (zero
-// diagonal, 0 <= D <= 2^22) is split into two fp16 pieces D = 2048 hi + lo,
-// both exact (< 2048), with fp32 accumulation of at most k terms each.
+// Put D'_ij = D_ij off the diagonal and D'_ii = -R_i, R_i = sum_j D_ij.  The
+// k-row gather of D' for token t is then minus the integer weight:
+//   V_ti = sum_{j in S_t} D'_ji = -w_ti,   w_ti = f_ti R_i - sum_{j in S_t} D_ji,
+// and with F the one-hot rows of the selected experts V = F D' is a matrix
+// product.  It is exact on the tensor cores: F is 0/1 in fp16 and D' is cut
+// into two fp16 pieces D' = 2048 hi + lo.  Off the diagonal 0 <= D <= T, so
+// hi = D >> 11 and lo = D & 2047; on the diagonal -R = 2048 a + b with a even
+// (a = -2 round(R / 4096)) and |b| <= 2048.  All pieces are exact in fp16
+// while R < 2^23 (R <= (E - 1) T, so T <= 66052), and k-term sums of them
+// stay below 2^24, exact in the fp32 accumulators.  With s = sigmoid(z),
+// S = sum_i s_i, SV = sum_i s_i V_ti and c = grad_scale d_scale / (m^2 k):
+//   A_t = sum_i p_ti w_ti = -SV / S,
+//   dz_ti = c/S s_i (1 - s_i) (w_ti - A_t) = s_i (1 - s_i) (c SV / S^2 - c/S V_ti).
 //
-// A persistent CTA owns a run of 128-token tiles of one problem.  Per tile:
-//   1. the four epilogue warps write F (128 x 128 fp16, K-major, 128-byte
-//      swizzle) from the selected-expert bytes;
-//   2. one thread issues 8 tcgen05.mma (M=128, N=256: hi | lo, K=16 each) into
-//      one of two TMEM accumulators, and commits to an mbarrier;
-//   3. meanwhile the epilogue of the previous tile runs: thread = token =
-//      TMEM lane.  Pass 1 streams the logits in 32 x 32 TMA boxes, forms s, S,
-//      sum s G and writes jac and G back into the accumulator columns; pass 2
-//      reads them again, writes dz into a swizzled staging box (plus the
-//      [i in S_t] term for the k selected experts) and stores it with TMA.
-// Tensor maps are 3-D [L][T][E], so boxes past the end of a problem are
-// zero-filled on load and dropped on store.
+// The pieces of D' come ready-made from the reduction kernel as the image of
+// the shared-memory operand B (dprime_pieces, 64 KB per problem).
+//
+// A persistent CTA takes a run of 128-token tiles of one problem:
+//   warp 0       allocates TMEM; one thread copies B in with one bulk copy and
+//                issues the MMAs V(tile) = F(tile) [hi | lo] (M = 128, N = 256,
+//                K = 128) into one of two accumulators, committed to an
+//                mbarrier per accumulator;
+//   warps 1-3    write F of the next tile (K-major, 128-byte swizzle) once
+//                the MMA of the previous one has read it;
+//   warps 4-19   the epilogue: warp w reads TMEM lanes 32 (w % 4) .. +31 (its
+//                32 tokens) and the 32 experts of chunk (w - 4) / 4.  Each owns
+//                a 32 x 32 logits box per tile, loaded by TMA two tiles ahead;
+//                pass 1 forms s, S and SV and writes s (1 - s) and V back into
+//                the accumulator (the reciprocals of four 1 + e^-|z| in (1, 2]
+//                come from one rcp of their product); the four warps of a
+//                token quadrant exchange their (S, SV) through their boxes;
+//                pass 2 writes dz into the box in place and a TMA store sends
+//                it to dlogits; once the store has read the box it takes the
+//                logits of the tile after next.
+// Tensor maps are 3-D [L][T][E]: rows past the end of a problem read as zero
+// and are dropped on store.
 #include <cuda_fp16.h>
 
 #include <climits>
@@ -35,49 +50,57 @@ namespace {
 
 constexpr int kE = 128;
 constexpr int kTileM = 128;
-constexpr int kEpiWarps = 8;                     // two per TMEM lane quadrant
-constexpr int kCtrlWarp = kEpiWarps;
-constexpr int kMmaThreads = (kEpiWarps + 1) * 32;
-constexpr int kEpiThreads = kEpiWarps * 32;
-constexpr int kBoxBytes = 32 * 128;              // 32 rows x 32 fp32
-constexpr int kAtomA = kTileM * 128;             // one 64-column K atom of A
-constexpr int kAtomB = 2 * kE * 128;             // one 64-column K atom of B (256 rows)
-constexpr int kBytesA = 2 * kAtomA;              // 32 KB
-constexpr int kBytesB = 2 * kAtomB;              // 64 KB
+constexpr int kEpiWarp0 = 4;                        // warps 4..19: w % 4 = TMEM quadrant
+constexpr int kEpiWarps = 16;                       // 4 quadrants x 4 expert chunks
+constexpr int kWarps = kEpiWarp0 + kEpiWarps;
+constexpr int kThreads = kWarps * 32;
+constexpr int kFWarp0 = 1, kFWarps = 3;             // builders of F
+constexpr int kFThreads = kFWarps * 32;
+constexpr int kBoxBytes = 32 * 128;                 // 32 rows x 32 fp32
+constexpr int kAtomA = kTileM * 128;                // one 64-column K atom of F
+constexpr int kAtomB = 2 * kE * 128;                // one 64-column K atom of B (256 rows)
+constexpr int kZBoxes = 2 * kEpiWarps;              // two tiles of boxes in flight
 constexpr int kOffB = 0;
-constexpr int kOffA = kOffB + kBytesB;           // one A buffer
-constexpr int kOffZ = kOffA + kBytesA;           // [chunk 4][quadrant 4] logits boxes
-constexpr int kOffO = kOffZ + 16 * kBoxBytes;    // [warp] dlogits staging box
-constexpr int kOffBar = kOffO + kEpiWarps * kBoxBytes;  // mma_done, zfull[16]
-constexpr int kOffScal = kOffBar + 8 * (1 + 16);        // tmem base, abort, last
-constexpr int kOffR = kOffScal + 16;                    // R_i [E] (64-bit)
-constexpr int kOffX = kOffR + 8 * kE;                   // exchange [half 2][token 128][3] fp32
-constexpr int kOffPart = kOffX + 2 * kTileM * 3 * 4;    // [kMmaThreads] fp64
-constexpr int kSmemMma = kOffPart + 8 * kMmaThreads + 1024;  // + alignment slack
-constexpr uint32_t kTmemCols = 512;              // two 256-column accumulators
+constexpr int kOffA = kOffB + 2 * kAtomB;           // 64 KB
+constexpr int kOffZ = kOffA + 2 * kAtomA;           // 96 KB
+constexpr int kOffBar = kOffZ + kZBoxes * kBoxBytes;  // 224 KB
+constexpr int kNumBars = 2 + 2 + 1 + 1 + kZBoxes;   // mma_done[2], acc_free[2], f_full, b_full, zfull[32]
+constexpr int kOffScal = kOffBar + 8 * kNumBars;    // tmem base, abort, last
+constexpr int kOffPart = kOffScal + 16;             // [kWarps] fp64
+constexpr int kSmemMma = kOffPart + 8 * kWarps + 1024;  // + alignment slack
+static_assert(kOffScal % 8 == 0 && kOffPart % 8 == 0, "alignment");
+static_assert(2 * kAtomB == kBImageBytes, "B image");
+static_assert(kSmemMma <= 232448, "shared memory");
+constexpr uint32_t kTmemCols = 512;                 // two 256-column accumulators
 constexpr float kLog2e = 1.4426950408889634f;
 
-__device__ __forceinline__ float sig_fast(float z) {
-    float e, r;
-    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(e) : "f"(z * -kLog2e));
-    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(1.0f + e));
-    return r;
+__device__ __forceinline__ float ex2_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
 }
 
-// Byte offset of element (row, k) of a K-major 128-byte-swizzled fp16 operand
-// with `rows` rows: K atoms of 64 columns, 128-byte rows, 16-byte chunks
-// XOR-ed with (row mod 8).
-__device__ __forceinline__ uint32_t sw128_fp16_offset(int row, int k, int rows) {
-    const int atom = k >> 6, kc = k & 63;
-    return (uint32_t)(atom * rows * 128 + row * 128 + ((((kc >> 3) ^ (row & 7))) << 4) + (kc & 7) * 2);
+__device__ __forceinline__ float rcp_approx(float x) {
+    float y;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__device__ __forceinline__ int atom_add_acq_rel(int *p, int v) {
+    int old;
+    asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
+
+__device__ __forceinline__ void named_sync(int id, int nthreads) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
 struct MmaArgs {
     const float *logits;
     const uint8_t *idx;
-    const int *D;
-    const int *counts;  // may be null: R then comes from the rows of D
-    int *n_zero;        // may be null
+    const unsigned char *bimg;  // [L][kBImageBytes]
+    int *n_zero;                // may be null
     int64_t T;
     int tiles_per_cta;
     float coef;
@@ -85,12 +108,27 @@ struct MmaArgs {
     double *partials;
     int *done;
     float *loss;
-    long long *origin_do;
     int *status;
 };
 
 template <int K>
-__global__ void __launch_bounds__(kMmaThreads, 1)
+__device__ __forceinline__ void load_sel(const uint8_t *p, uint32_t (&r)[2]) {
+    r[0] = r[1] = 0u;
+    if (K == 8) {
+        const uint2 v = __ldg(reinterpret_cast<const uint2 *>(p));
+        r[0] = v.x;
+        r[1] = v.y;
+    } else if (K == 4) {
+        r[0] = __ldg(reinterpret_cast<const uint32_t *>(p));
+    } else if (K == 2) {
+        r[0] = __ldg(reinterpret_cast<const uint16_t *>(p));
+    } else {
+        r[0] = __ldg(p);
+    }
+}
+
+template <int K>
+__global__ void __launch_bounds__(kThreads, 1)
 loss_mma_kernel(const __grid_constant__ CUtensorMap zmap, const __grid_constant__ CUtensorMap dzmap,
                 const MmaArgs a) {
     extern __shared__ unsigned char smem_raw[];
@@ -99,14 +137,15 @@ loss_mma_kernel(const __grid_constant__ CUtensorMap zmap, const __grid_constant_
     unsigned char *sB = smem + kOffB;
     unsigned char *sA = smem + kOffA;
     unsigned char *sZ = smem + kOffZ;
-    unsigned char *sO = smem + kOffO;
-    uint64_t *mma_done = reinterpret_cast<uint64_t *>(smem + kOffBar);      // one phase per tile
-    uint64_t *zfull = mma_done + 1;                                          // [chunk][quadrant]
-    float *s_x = reinterpret_cast<float *>(smem + kOffX);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kOffBar);
+    uint64_t *mma_done = bars;      // [accumulator]: phase n = n-th MMA into it done
+    uint64_t *acc_free = bars + 2;  // [accumulator]: the epilogue has read it
+    uint64_t *f_full = bars + 4;    // F of the next tile written
+    uint64_t *b_full = bars + 5;    // B copied in
+    uint64_t *zfull = bars + 6;     // [set][epilogue warp]: logits box loaded
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + kOffScal);
     volatile int *s_abort = reinterpret_cast<volatile int *>(smem + kOffScal + 4);
     int *s_last = reinterpret_cast<int *>(smem + kOffScal + 8);
-    unsigned long long *s_R = reinterpret_cast<unsigned long long *>(smem + kOffR);
     double *s_part = reinterpret_cast<double *>(smem + kOffPart);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -118,338 +157,323 @@ loss_mma_kernel(const __grid_constant__ CUtensorMap zmap, const __grid_constant_
     const int nt = te > tb ? te - tb : 0;
 
     if (threadIdx.x == 0) {
-        mbar_init(&mma_done[0], 1);
-        for (int i = 0; i < 16; ++i) mbar_init(&zfull[i], 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&mma_done[i], 1);
+            mbar_init(&acc_free[i], kEpiWarps / 2);
+        }
+        mbar_init(f_full, kFWarps);
+        mbar_init(b_full, 1);
+        for (int i = 0; i < kZBoxes; ++i) mbar_init(&zfull[i], 1);
         *s_abort = 0;
         fence_barrier_init();
     }
-    if (threadIdx.x < kE) s_R[threadIdx.x] = 0ull;
-    if (warp == kCtrlWarp) tmem_alloc(tmem_slot, kTmemCols);
+    if (warp == 0) tmem_alloc(tmem_slot, kTmemCols);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    // The logits are an input of the whole path: start the first tile's boxes
-    // before waiting for the previous kernels.
-    // epilogue warp w: TMEM lane quadrant q = w % 4 (tokens 32q..), half h = w / 4
-    // (experts 64h .. 64h+63, chunks 2h and 2h+1); it loads and consumes the
-    // logits boxes (chunk, q) of its chunks.
-    const int quad = warp & 3, half = warp >> 2;
-    auto issue_z = [&](int tile, int chunk) {
-        uint64_t *bar = &zfull[chunk * 4 + quad];
-        mbar_arrive_expect_tx(bar, kBoxBytes);
-        tma_load_3d(sZ + (chunk * 4 + quad) * kBoxBytes, &zmap, 32 * chunk,
-                    tile * kTileM + 32 * quad, layer, bar);
+    // epilogue warps: group g = tiles of parity g (accumulator g, box set g);
+    // within it quadrant q (tokens 32q ..) and chunk pair p (experts 64p ..)
+    const bool epi = warp >= kEpiWarp0;
+    const int ew = epi ? warp - kEpiWarp0 : 0;
+    const int group = ew >> 3, quad = warp & 3, pair = (ew >> 2) & 1;
+    auto box_id = [&](int cc) { return group * kEpiWarps + (2 * pair + cc) * 4 + quad; };
+    auto issue_z = [&](int m) {  // tile tb + m (parity = group) into this warp's two boxes
+#pragma unroll
+        for (int cc = 0; cc < 2; ++cc) {
+            uint64_t *bar = &zfull[box_id(cc)];
+            mbar_arrive_expect_tx(bar, kBoxBytes);
+            tma_load_3d(sZ + (size_t)box_id(cc) * kBoxBytes, &zmap, 32 * (2 * pair + cc),
+                        (tb + m) * kTileM + 32 * quad, layer, bar);
+        }
     };
-    if (warp < kEpiWarps && lane == 0 && nt > 0) {
+    // The logits are an input of the whole path: each group's first tile is
+    // requested before waiting for the previous kernels.
+    int z_issued = 0;  // tiles of this group requested (lane 0)
+    if (epi && lane == 0) {
         prefetch_tensormap(&zmap);
         prefetch_tensormap(&dzmap);
-        issue_z(tb, 2 * half);
-        issue_z(tb, 2 * half + 1);
-    }
-
-    pdl_wait();  // D, the counts and the selected experts come from the previous kernels
-
-    // B = [hi rows 0..127 | lo rows 128..255] x K 128, from the rows of D
-    // (D symmetric: row n of D is column n); R_i = sum_j D_ij alongside.
-    const int *Dl = a.D + (int64_t)layer * kE * kE;
-    constexpr int kItems = kE * (kE / 8);  // 16-byte fp16 chunks of one B half
-    constexpr int kPer = (kItems + kMmaThreads - 1) / kMmaThreads;
-    int4 dv[kPer][2];
-#pragma unroll
-    for (int u = 0; u < kPer; ++u) {  // all loads first: one round trip
-        const int item = threadIdx.x + u * kMmaThreads;
-        if (item < kItems) {
-            const int n = item >> 4, k0 = (item & 15) * 8;
-            dv[u][0] = __ldg(reinterpret_cast<const int4 *>(Dl + n * kE + k0));
-            dv[u][1] = __ldg(reinterpret_cast<const int4 *>(Dl + n * kE + k0 + 4));
+        if (group < nt) {
+            issue_z(group);
+            z_issued = 1;
         }
     }
-#pragma unroll
-    for (int u = 0; u < kPer; ++u) {
-        const int item = threadIdx.x + u * kMmaThreads;
-        if (item >= kItems) break;
-        const int n = item >> 4, k0 = (item & 15) * 8;
-        const int4 v0 = dv[u][0], v1 = dv[u][1];
-        const int d[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
-        __align__(16) __half hi[8], lo[8];
-        long long rs = 0;
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-            hi[q] = __int2half_rn(d[q] >> 11);
-            lo[q] = __int2half_rn(d[q] & 2047);
-            rs += d[q];
-        }
-        *reinterpret_cast<uint4 *>(sB + sw128_fp16_offset(n, k0, 2 * kE)) =
-            *reinterpret_cast<const uint4 *>(hi);
-        *reinterpret_cast<uint4 *>(sB + sw128_fp16_offset(kE + n, k0, 2 * kE)) =
-            *reinterpret_cast<const uint4 *>(lo);
-        if (!a.counts) atomicAdd(&s_R[n], (unsigned long long)rs);
-    }
-    if (a.counts && threadIdx.x < kE) {
-        const long long nn = a.counts[(int64_t)layer * kE + threadIdx.x];
-        s_R[threadIdx.x] = (unsigned long long)((long long)(kE - 2 * K) * nn + T * (long long)K);
-        if (a.n_zero && blockIdx.x == 0) a.n_zero[(int64_t)layer * kE + threadIdx.x] = 0;
-    }
-    fence_proxy_async_smem();
-    __syncthreads();
-    if (threadIdx.x < kE) {
-        const long long r = (long long)s_R[threadIdx.x];
-        if (r > INT_MAX || r < 0) atomicOr(a.status, kDevOverflow);
-    }
 
-    // kind::f16 instruction descriptor: fp32 accumulate, fp16 A and B, both
-    // K-major, N = 256, M = 128.
-    const uint32_t idesc = (1u << 4) | ((uint32_t)(2 * kE / 8) << 17) | ((uint32_t)(kTileM / 16) << 24);
-    const uint32_t sA_u32 = smem_u32(sA), sB_u32 = smem_u32(sB);
+    pdl_wait();  // the image of D', D and the selected experts come from the previous kernels
 
-    double tok_sum = 0.0;
-    // selected experts of this thread's token (row 32 quad + lane) in the
-    // current and the previous tile, and the raw bytes of the next tile
-    int js[K], js_prev[K];
-    uint32_t jn[2] = {0u, 0u};
-    bool valid_prev = false;
-    const int row = 32 * quad + lane;
+    float tok_sum = 0.0f;  // sum of A_t over this thread's tokens (at most a few tiles)
+    if (warp == 0) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            // kind::f16: fp32 accumulate, fp16 A and B, both K-major, N = 256, M = 128
+            const uint32_t idesc =
+                (1u << 4) | ((uint32_t)(2 * kE / 8) << 17) | ((uint32_t)(kTileM / 16) << 24);
+            const uint32_t sA_u32 = smem_u32(sA), sB_u32 = smem_u32(sB);
+            mbar_arrive_expect_tx(b_full, kBImageBytes);
+            const unsigned char *img = a.bimg + (size_t)layer * kBImageBytes;
 #pragma unroll
-    for (int q = 0; q < K; ++q) js[q] = js_prev[q] = 0;
-    auto load_idx_raw = [&](int tile, uint32_t (&r)[2]) {
-        const int64_t tt = (int64_t)tile * kTileM + row;
-        r[0] = r[1] = 0u;
-        if (tt < T) {
-            const uint8_t *ip = a.idx + ((int64_t)layer * T + tt) * K;
-            if (K == 8) {
-                const uint2 v = __ldg(reinterpret_cast<const uint2 *>(ip));
-                r[0] = v.x;
-                r[1] = v.y;
-            } else if (K == 4) {
-                r[0] = __ldg(reinterpret_cast<const uint32_t *>(ip));
-            } else if (K == 2) {
-                r[0] = __ldg(reinterpret_cast<const uint16_t *>(ip));
-            } else {
-                r[0] = __ldg(ip);
-            }
-        }
-    };
-    if (warp < kEpiWarps && nt > 0) load_idx_raw(tb, jn);
-
-    for (int it = 0; it <= nt; ++it) {
-        bool valid = false;
-        if (warp < kEpiWarps) {
-            // the MMA of the previous tile is done: A is free, its accumulator full
-            if (it >= 1 && !mbar_wait(&mma_done[0], (uint32_t)((it - 1) & 1), a.status)) *s_abort = 1;
-            tc_fence_after();
-            if (it < nt) {
-                valid = (int64_t)(tb + it) * kTileM + row < T;
+            for (int q = 0; q < 4; ++q)
+                bulk_load(sB + q * (kBImageBytes / 4), img + q * (kBImageBytes / 4), kBImageBytes / 4,
+                          b_full);
+            const bool have_b = mbar_wait(b_full, 0u, a.status);
+            if (!have_b) *s_abort = 1;
+            int issued = 0;
+            for (int m = 0; m < nt && have_b; ++m) {
+                const int buf = m & 1;
+                bool ok = mbar_wait(f_full, (uint32_t)m & 1u, a.status);
+                if (ok && m >= 2)
+                    ok = mbar_wait(&acc_free[buf], (uint32_t)((m >> 1) - 1) & 1u, a.status);
+                if (!ok) *s_abort = 1;
+                if (*s_abort) break;
+                tc_fence_after();
+                const uint32_t d_tmem = tmem + (uint32_t)(buf * 2 * kE);
 #pragma unroll
-                for (int q = 0; q < K; ++q) js[q] = (jn[q / 4] >> (8 * (q % 4))) & 0xff;
-                if (it + 1 < nt) load_idx_raw(tb + it + 1, jn);
-                // 1. F of tile it: half h writes K atom h of the token's row
-                unsigned char *arow = sA + half * kAtomA + row * 128;
-#pragma unroll
-                for (int q = 0; q < 8; ++q)  // chunk order rotated by row: conflict-free
-                    *reinterpret_cast<uint4 *>(arow + ((q ^ (row & 7)) << 4)) = make_uint4(0, 0, 0, 0);
-                if (valid) {
-                    const __half one = __float2half(1.0f);
-#pragma unroll
-                    for (int q = 0; q < K; ++q)
-                        if ((js[q] >> 6) == half)
-                            *reinterpret_cast<__half *>(sA + sw128_fp16_offset(row, js[q], kTileM)) = one;
+                for (int kk = 0; kk < kE / 16; ++kk) {
+                    const uint32_t koff = (uint32_t)((kk & 3) * 32);
+                    const uint64_t adesc = umma_desc_sw128(sA_u32 + (kk >> 2) * kAtomA + koff);
+                    const uint64_t bdesc = umma_desc_sw128(sB_u32 + (kk >> 2) * kAtomB + koff);
+                    umma_f16(d_tmem, adesc, bdesc, idesc, kk > 0 ? 1u : 0u);
                 }
-                fence_proxy_async_smem();
+                umma_commit(&mma_done[buf]);
+                issued = m + 1;
             }
+            // the tensor cores must be done with TMEM before it is released
+            if (issued > 0)
+                mbar_wait(&mma_done[(issued - 1) & 1], (uint32_t)((issued - 1) >> 1) & 1u, a.status);
+            if (!have_b) mbar_wait(b_full, 0u, a.status);  // no copy may outlive the CTA
         }
-        tc_fence_before();
-        asm volatile("bar.sync 1, %0;" ::"n"(kMmaThreads) : "memory");
-        tc_fence_after();
-        if (*s_abort) break;
-        // 2. the tensor cores: G(it) = F(it) [D_hi | D_lo] into accumulator it & 1
-        if (it < nt && warp == kCtrlWarp && lane == 0) {
-            const uint32_t d_tmem = tmem + (uint32_t)((it & 1) * 2 * kE);
+        __syncwarp();
+    } else if (warp < kEpiWarp0) {
+        // ------------------------------------------------------------ F builders
+        const int ft = threadIdx.x - kFWarp0 * 32;
+        constexpr int kRows = (kTileM + kFThreads - 1) / kFThreads;
+        uint32_t sel[kRows][2];
+        auto load_rows = [&](int m) {
 #pragma unroll
-            for (int kk = 0; kk < kE / 16; ++kk) {
-                const uint32_t koff = (uint32_t)((kk & 3) * 32);
-                const uint64_t adesc = umma_desc_sw128(sA_u32 + (kk >> 2) * kAtomA + koff);
-                const uint64_t bdesc = umma_desc_sw128(sB_u32 + (kk >> 2) * kAtomB + koff);
-                umma_f16(d_tmem, adesc, bdesc, idesc, kk > 0 ? 1u : 0u);
+            for (int i = 0; i < kRows; ++i) {
+                const int r = ft + i * kFThreads;
+                const int64_t t = (int64_t)(tb + m) * kTileM + r;
+                sel[i][0] = sel[i][1] = 0u;
+                if (r < kTileM && t < T) load_sel<K>(a.idx + ((int64_t)layer * T + t) * K, sel[i]);
             }
-            umma_commit(&mma_done[0]);
-        }
-        // 3. epilogue of tile it - 1 on this warp's half of the experts
-        if (it >= 1 && warp < kEpiWarps) {
-            const int pt = it - 1, pbuf = pt & 1;
-            const int ptile = tb + pt;
+        };
+        if (nt > 0) load_rows(0);
+        // the counts accumulator of the signatures kernel is read (by the
+        // reduction): clear it for the next call
+        if (a.n_zero && blockIdx.x == 0)
+            for (int i = ft; i < kE; i += kFThreads) a.n_zero[(int64_t)layer * kE + i] = 0;
+        const __half one = __float2half(1.0f);
+        for (int m = 0; m < nt; ++m) {
+            // F(m - 1) has been read by its MMA
             bool ok = true;
-            const uint32_t tl = tmem + ((uint32_t)(32 * quad) << 16) + (uint32_t)(pbuf * 2 * kE);
-            float S0 = 0.f, S1 = 0.f, G0 = 0.f, G1 = 0.f;
-            float zsel[K];
+            if (m >= 1)
+                ok = mbar_wait(&mma_done[(m - 1) & 1], (uint32_t)((m - 1) >> 1) & 1u, a.status);
+            if (!ok) *s_abort = 1;
+            if (*s_abort) break;
 #pragma unroll
-            for (int q = 0; q < K; ++q) zsel[q] = 0.0f;
-            // pass 1
+            for (int i = 0; i < kRows; ++i) {
+                const int r = ft + i * kFThreads;
+                if (r >= kTileM) break;
+#pragma unroll
+                for (int at = 0; at < 2; ++at)
+#pragma unroll
+                    for (int q = 0; q < 8; ++q)
+                        *reinterpret_cast<uint4 *>(sA + at * kAtomA + r * 128 + ((q ^ (r & 7)) << 4)) =
+                            make_uint4(0, 0, 0, 0);
+                const int64_t t = (int64_t)(tb + m) * kTileM + r;
+                if (t < T) {
+#pragma unroll
+                    for (int q = 0; q < K; ++q) {
+                        const int j = (sel[i][q / 4] >> (8 * (q % 4))) & 0xff;
+                        *reinterpret_cast<__half *>(sA + sw128_k16_offset(r, j, kTileM)) = one;
+                    }
+                }
+            }
+            if (m + 1 < nt) load_rows(m + 1);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(f_full);
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue
+        const int row = 32 * quad + lane;
+        const uint32_t tl0 = tmem + ((uint32_t)(32 * quad) << 16) + (uint32_t)(group * 2 * kE) +
+                             (uint32_t)(64 * pair);
+        int z_done = 0;  // tiles of this group waited for (lane 0)
+        for (int m = group; m < nt; m += 2) {
+            const uint32_t ph = (uint32_t)(m >> 1) & 1u;
+            bool ok = mbar_wait(&mma_done[group], ph, a.status);
+            if (ok) ok = mbar_wait(&zfull[box_id(0)], ph, a.status) && mbar_wait(&zfull[box_id(1)], ph, a.status);
+            if (ok) z_done = (m >> 1) + 1;
+            if (!ok) *s_abort = 1;
+            ok = __all_sync(kFull, ok && !*s_abort);
+            tc_fence_after();
+            float S = 0.f, SV = 0.f;
+            if (ok) {
+                // pass 1: s, S, SV; s (1 - s) and V back into the accumulator
+#pragma unroll 1
+                for (int cc = 0; cc < 2; ++cc) {
+                    const unsigned char *zrow = sZ + (size_t)box_id(cc) * kBoxBytes + lane * 128;
+                    const uint32_t tl = tl0 + 32 * cc;
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        uint32_t hi[16], lo[16];
+                        tmem_ld16(tl + 16 * h, hi);
+                        tmem_ld16(tl + kE + 16 * h, lo);
+                        float z[16];
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            const float4 v = *reinterpret_cast<const float4 *>(
+                                zrow + (((4 * h + q) ^ (lane & 7)) << 4));
+                            z[4 * q] = v.x;
+                            z[4 * q + 1] = v.y;
+                            z[4 * q + 2] = v.z;
+                            z[4 * q + 3] = v.w;
+                        }
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int g = 0; g < 4; ++g) {
+                            float ee[4], dd[4], inv[4];
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                ee[i] = ex2_approx(fabsf(z[4 * g + i]) * -kLog2e);
+                                dd[i] = 1.0f + ee[i];
+                            }
+                            const float p01 = dd[0] * dd[1], p012 = p01 * dd[2];
+                            float r = rcp_approx(p012 * dd[3]);
+                            inv[3] = r * p012;
+                            r *= dd[3];
+                            inv[2] = r * p01;
+                            r *= dd[2];
+                            inv[1] = r * dd[0];
+                            inv[0] = r * dd[1];
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                const int e = 4 * g + i;
+                                const float V = fmaf(__uint_as_float(hi[e]), 2048.0f, __uint_as_float(lo[e]));
+                                const float s = (z[e] >= 0.0f ? 1.0f : ee[i]) * inv[i];
+                                S += s;
+                                SV = fmaf(s, V, SV);
+                                hi[e] = __float_as_uint(ee[i] * inv[i] * inv[i]);
+                                lo[e] = __float_as_uint(V);
+                            }
+                        }
+                        tmem_st16(tl + 16 * h, hi);
+                        tmem_st16(tl + kE + 16 * h, lo);
+                    }
+                }
+                tmem_wait_st();
+            }
+            // exchange with the other chunk pair of the quadrant through the
+            // first 16 bytes of this row of the pair's first box
+            unsigned char *myrow = sZ + (size_t)box_id(0) * kBoxBytes + lane * 128;
+            float *slot = reinterpret_cast<float *>(myrow + ((lane & 7) << 4));
+            slot[0] = S;
+            slot[1] = SV;
+            slot[2] = ok ? 1.0f : 0.0f;
+            named_sync(1 + 4 * group + quad, 64);
+            float St = 0.f, SVt = 0.f;
+            bool all_ok = true;
+#pragma unroll
+            for (int pp = 0; pp < 2; ++pp) {
+                const float *o = reinterpret_cast<const float *>(
+                    sZ + (size_t)(group * kEpiWarps + (2 * pp) * 4 + quad) * kBoxBytes + lane * 128 +
+                    ((lane & 7) << 4));
+                St += o[0];
+                SVt += o[1];
+                all_ok = all_ok && o[2] != 0.0f;
+            }
+            all_ok = __all_sync(kFull, all_ok);
+            if (!all_ok) break;  // the same decision in both warps of the quadrant
+            named_sync(1 + 4 * group + quad, 64);
+            const float cs = a.coef / St;
+            const float csA = cs * (SVt / St);
+            if (pair == 0 && (int64_t)(tb + m) * kTileM + row < T) tok_sum -= SVt / St;
+            // pass 2: dz into the boxes, in place
 #pragma unroll 1
             for (int cc = 0; cc < 2; ++cc) {
-                const int c = 2 * half + cc;
-                ok = mbar_wait(&zfull[c * 4 + quad], (uint32_t)pt & 1u, a.status);
-                if (!ok) break;
-                uint32_t hi[32], lo[32];
-                tmem_ld32(tl + 32 * c, hi);
-                tmem_ld32(tl + kE + 32 * c, lo);
-                const unsigned char *zrow = sZ + (c * 4 + quad) * kBoxBytes + lane * 128;
-                float z[32];
+                unsigned char *zrow = sZ + (size_t)box_id(cc) * kBoxBytes + lane * 128;
+                const uint32_t tl = tl0 + 32 * cc;
 #pragma unroll
-                for (int q = 0; q < 8; ++q) {
-                    const float4 v =
-                        *reinterpret_cast<const float4 *>(zrow + ((q ^ (lane & 7)) << 4));
-                    z[4 * q] = v.x;
-                    z[4 * q + 1] = v.y;
-                    z[4 * q + 2] = v.z;
-                    z[4 * q + 3] = v.w;
-                }
+                for (int h = 0; h < 2; ++h) {
+                    uint32_t jac[16], vv[16];
+                    tmem_ld16(tl + 16 * h, jac);
+                    tmem_ld16(tl + kE + 16 * h, vv);
+                    tmem_wait_ld();
 #pragma unroll
-                for (int q = 0; q < K; ++q)
-                    if ((js_prev[q] >> 5) == c) {
-                        const int e = js_prev[q] & 31;
-                        zsel[q] = *reinterpret_cast<const float *>(
-                            zrow + ((((e >> 2) ^ (lane & 7))) << 4) + (e & 3) * 4);
-                    }
-                tmem_wait_ld();
-#pragma unroll
-                for (int e = 0; e < 32; e += 2) {
-                    const float Ga = fmaf(__uint_as_float(hi[e]), 2048.0f, __uint_as_float(lo[e]));
-                    const float Gb =
-                        fmaf(__uint_as_float(hi[e + 1]), 2048.0f, __uint_as_float(lo[e + 1]));
-                    const float sa = sig_fast(z[e]), sb = sig_fast(z[e + 1]);
-                    S0 += sa;
-                    S1 += sb;
-                    G0 = fmaf(sa, Ga, G0);
-                    G1 = fmaf(sb, Gb, G1);
-                    hi[e] = __float_as_uint(fmaf(-sa, sa, sa));
-                    hi[e + 1] = __float_as_uint(fmaf(-sb, sb, sb));
-                    lo[e] = __float_as_uint(Ga);
-                    lo[e + 1] = __float_as_uint(Gb);
-                }
-                tmem_st32(tl + 32 * c, hi);
-                tmem_st32(tl + kE + 32 * c, lo);
-                // every lane has consumed its row of the box: load the next tile's box
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0 && pt + 1 < nt) issue_z(ptile + 1, c);
-            }
-            tmem_wait_st();
-            // the selected experts in this half: sum s_j R_j, and jac_j R_j for dz
-            float SRv = 0.0f, patch[K];
-#pragma unroll
-            for (int q = 0; q < K; ++q) {
-                const bool mine = (js_prev[q] >> 6) == half;
-                const float sj = sig_fast(zsel[q]);
-                const float rj = (float)(long long)s_R[js_prev[q]];
-                SRv += mine ? sj * rj : 0.0f;
-                patch[q] = fmaf(-sj, sj, sj) * rj;
-            }
-            // exchange the half sums of every token; add them in a fixed order
-            float *xr = s_x + (half * kTileM + row) * 3;
-            xr[0] = S0 + S1;
-            xr[1] = G0 + G1;
-            xr[2] = SRv;
-            asm volatile("bar.sync 2, %0;" ::"n"(kEpiThreads) : "memory");
-            const float *x0 = s_x + row * 3, *x1 = s_x + (kTileM + row) * 3;
-            const float S = x0[0] + x1[0];
-            const float A = ((x0[2] + x1[2]) - (x0[1] + x1[1])) / S;
-            const float cs = a.coef / S;
-            asm volatile("bar.sync 2, %0;" ::"n"(kEpiThreads) : "memory");
-            if (half == 0 && valid_prev && ok) tok_sum += (double)A;
-            // pass 2
-#pragma unroll 1
-            for (int cc = 0; cc < 2 && ok; ++cc) {
-                const int c = 2 * half + cc;
-                uint32_t jac[32], gg[32];
-                tmem_ld32(tl + 32 * c, jac);
-                tmem_ld32(tl + kE + 32 * c, gg);
-                if (lane == 0) bulk_wait_read<0>();
-                __syncwarp();
-                tmem_wait_ld();
-                unsigned char *orow = sO + warp * kBoxBytes + lane * 128;
-#pragma unroll
-                for (int q = 0; q < 8; ++q) {
-                    float4 v;
-                    v.x = -cs * __uint_as_float(jac[4 * q]) * (__uint_as_float(gg[4 * q]) + A);
-                    v.y = -cs * __uint_as_float(jac[4 * q + 1]) * (__uint_as_float(gg[4 * q + 1]) + A);
-                    v.z = -cs * __uint_as_float(jac[4 * q + 2]) * (__uint_as_float(gg[4 * q + 2]) + A);
-                    v.w = -cs * __uint_as_float(jac[4 * q + 3]) * (__uint_as_float(gg[4 * q + 3]) + A);
-                    *reinterpret_cast<float4 *>(orow + ((q ^ (lane & 7)) << 4)) = v;
-                }
-#pragma unroll
-                for (int q = 0; q < K; ++q) {
-                    if (valid_prev && (js_prev[q] >> 5) == c) {
-                        const int e = js_prev[q] & 31;
-                        float *p = reinterpret_cast<float *>(orow + ((((e >> 2) ^ (lane & 7))) << 4)) + (e & 3);
-                        *p += cs * patch[q];
+                    for (int q = 0; q < 4; ++q) {
+                        float4 o;
+                        o.x = __uint_as_float(jac[4 * q]) * fmaf(-cs, __uint_as_float(vv[4 * q]), csA);
+                        o.y = __uint_as_float(jac[4 * q + 1]) * fmaf(-cs, __uint_as_float(vv[4 * q + 1]), csA);
+                        o.z = __uint_as_float(jac[4 * q + 2]) * fmaf(-cs, __uint_as_float(vv[4 * q + 2]), csA);
+                        o.w = __uint_as_float(jac[4 * q + 3]) * fmaf(-cs, __uint_as_float(vv[4 * q + 3]), csA);
+                        *reinterpret_cast<float4 *>(zrow + (((4 * h + q) ^ (lane & 7)) << 4)) = o;
                     }
                 }
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0) {
-                    tma_store_3d(&dzmap, sO + warp * kBoxBytes, 32 * c, ptile * kTileM + 32 * quad,
-                                 layer);
-                    bulk_commit_group();
+            }
+            // the accumulator may take the MMA of tile m + 2
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&acc_free[group]);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+#pragma unroll
+                for (int cc = 0; cc < 2; ++cc)
+                    tma_store_3d(&dzmap, sZ + (size_t)box_id(cc) * kBoxBytes, 32 * (2 * pair + cc),
+                                 (tb + m) * kTileM + 32 * quad, layer);
+                bulk_commit_group();
+                // the boxes take this group's next tile once the stores have read them
+                if (m + 2 < nt) {
+                    bulk_wait_read<0>();
+                    issue_z(m + 2);
+                    ++z_issued;
                 }
             }
-            if (!ok) *s_abort = 1;
+            __syncwarp();
         }
-#pragma unroll
-        for (int q = 0; q < K; ++q) js_prev[q] = js[q];
-        valid_prev = valid;
+        if (lane == 0) {
+            bulk_wait_all<0>();  // dz stores complete
+            // loads requested but not consumed (only after a failed wait)
+            for (int j = z_done; j < z_issued; ++j) {
+                mbar_wait(&zfull[box_id(0)], (uint32_t)j & 1u, a.status);
+                mbar_wait(&zfull[box_id(1)], (uint32_t)j & 1u, a.status);
+            }
+        }
+        __syncwarp();
     }
 
-    // drain: stores complete, TMEM released
-    if (warp < kEpiWarps && lane == 0) bulk_wait_all<0>();
+    // TMEM released once every role is done with it
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == kCtrlWarp) tmem_dealloc(tmem, kTmemCols);
+    if (warp == 0) tmem_dealloc(tmem, kTmemCols);
 
-    // CTA partial in a fixed order (fp64 adds are slow on this part: a
-    // shuffle tree per warp, then the warp sums), then the last CTA
+    // CTA partial in a fixed order: a shuffle tree per warp, then the warp sums
+    double tok = (double)tok_sum;
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) tok_sum += __shfl_xor_sync(kFull, tok_sum, off);
-    if (lane == 0) s_part[warp] = tok_sum;
+    for (int off = 16; off > 0; off >>= 1) tok += __shfl_xor_sync(kFull, tok, off);
+    if (lane == 0) s_part[warp] = tok;
     __syncthreads();
-    if (threadIdx.x == 0) {
-        double sum = 0.0;
-        for (int i = 0; i < kMmaThreads / 32; ++i) sum += s_part[i];
-        a.partials[(int64_t)layer * gridDim.x + blockIdx.x] = sum;
-        __threadfence();
-        *s_last = (atomicAdd(&a.done[layer], 1) == (int)gridDim.x - 1);
+    if (warp == 0) {
+        double v = lane < kWarps ? s_part[lane] : 0.0;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(kFull, v, off);
+        if (lane == 0) {
+            a.partials[(int64_t)layer * gridDim.x + blockIdx.x] = v;
+            // release: the partial is visible to the CTA that sees the last count
+            *s_last = (atom_add_acq_rel(&a.done[layer], 1) == (int)gridDim.x - 1);
+        }
     }
     __syncthreads();
     if (!*s_last) return;
     __threadfence();
-    {
-        const double sum = block_sum_fixed(a.partials + (int64_t)layer * gridDim.x, gridDim.x,
-                                           s_part, 256);
-        if (threadIdx.x == 0) {
+    if (warp == 0) {
+        const double sum = warp_sum_fixed(a.partials + (int64_t)layer * gridDim.x, gridDim.x);
+        if (lane == 0) {
             a.loss[layer] = (float)(sum * a.scale);
             a.done[layer] = 0;
-        }
-    }
-    if (a.origin_do) {
-        long long o = 0;
-        for (int e = threadIdx.x; e < kE * kE; e += kMmaThreads) {
-            if (e / kE != e % kE) {
-                const long long d = Dl[e];
-                o += d * d;
-            }
-        }
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) o += __shfl_xor_sync(kFull, o, off);
-        __syncthreads();
-        long long *s_o = reinterpret_cast<long long *>(s_part);
-        if (lane == 0) s_o[warp] = o;
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            long long sum = 0;
-            for (int q = 0; q < kMmaThreads / 32; ++q) sum += s_o[q];
-            a.origin_do[layer] = sum;
         }
     }
 }
@@ -472,7 +496,7 @@ cudaError_t run_mma(const CUtensorMap &zmap, const CUtensorMap &dzmap, const Mma
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)gx, (unsigned)L);
-    cfg.blockDim = dim3(kMmaThreads);
+    cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = kSmemMma;
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
@@ -489,7 +513,9 @@ bool loss_mma_supported(const Problem &p, int gate, const float *logits, const i
                         const float *dlogits) {
     const bool k_ok = p.k == 1 || p.k == 2 || p.k == 4 || p.k == 8;
     auto al = [](const void *q) { return reinterpret_cast<uintptr_t>(q) % 16 == 0; };
-    return p.E == kE && gate == 0 && k_ok && dlogits != nullptr && p.T <= (1 << 22) && al(logits) &&
+    // R_i <= (E - 1) T must stay below 2^23 for the two-piece split of D'
+    const bool t_ok = (int64_t)(kE - 1) * p.T < (int64_t)(1 << 23);
+    return p.E == kE && gate == 0 && k_ok && dlogits != nullptr && t_ok && al(logits) &&
            al(dlogits) && al(D);
 }
 
@@ -502,10 +528,10 @@ int loss_mma_ctas_per_problem(const Problem &p) {
     return (tiles + per - 1) / per;
 }
 
-cudaError_t launch_loss_mma(const float *logits, const uint8_t *idx, const int *D, const int *counts,
-                            int *n_zero, const Problem &p, float d_scale, float grad_scale,
-                            float *loss, long long *origin_do, float *dlogits, double *partials,
-                            int *done, int *status, cudaStream_t s) {
+cudaError_t launch_loss_mma(const float *logits, const uint8_t *idx, const unsigned char *bimg, int *n_zero, const Problem &p, float d_scale,
+                            float grad_scale, float *loss, float *dlogits,
+                            double *partials, int *done, int *status, cudaStream_t s) {
+    if (!bimg) return cudaErrorInvalidValue;
     CUtensorMap zmap, dzmap;
     if (!encode_tensor_map_3d_f32(&zmap, logits, (uint64_t)p.L, (uint64_t)p.T, (uint64_t)kE, 32) ||
         !encode_tensor_map_3d_f32(&dzmap, dlogits, (uint64_t)p.L, (uint64_t)p.T, (uint64_t)kE, 32))
@@ -516,8 +542,7 @@ cudaError_t launch_loss_mma(const float *logits, const uint8_t *idx, const int *
     MmaArgs args;
     args.logits = logits;
     args.idx = idx;
-    args.D = D;
-    args.counts = counts;
+    args.bimg = bimg;
     args.n_zero = n_zero;
     args.T = p.T;
     args.tiles_per_cta = (tiles + gx - 1) / gx;
@@ -526,7 +551,6 @@ cudaError_t launch_loss_mma(const float *logits, const uint8_t *idx, const int *
     args.partials = partials;
     args.done = done;
     args.loss = loss;
-    args.origin_do = origin_do;
     args.status = status;
     switch (p.k) {
         case 1: return run_mma<1>(zmap, dzmap, args, gx, p.L, s);

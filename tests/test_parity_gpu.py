@@ -242,19 +242,23 @@ def test_repeated_calls_reuse_workspace(dl):
     assert dl.device_status(out.workspace) == 0
 
 
-@pytest.mark.parametrize("T,k,L", [(65536, 8, 1), (4096 + 33, 4, 2), (300, 1, 1), (1000, 2, 3)])
-def test_tcgen05_loss_kernel(dl, monkeypatch, T, k, L):
-    """The tensor-core gradient pass, chosen by DOLOSS_LOSS_KERNEL=tcgen05."""
+@pytest.mark.parametrize("T,k,L", [(65536, 8, 1), (4096 + 33, 4, 2), (300, 1, 1), (1000, 2, 3),
+                                   (66052, 8, 1), (128 * 5 + 1, 8, 2)])
+def test_tcgen05_and_alu_loss_kernels_agree(dl, monkeypatch, T, k, L):
+    """The tensor-core gradient pass (default at E = 128) against the ALU one
+    (DOLOSS_LOSS_KERNEL=alu), and both against the oracle at small T."""
     z = workloads.random_logits(T, 128, L=L, seed=T + k, ties=T < 2000)
-    monkeypatch.setenv("DOLOSS_LOSS_KERNEL", "tcgen05")
+    monkeypatch.delenv("DOLOSS_LOSS_KERNEL", raising=False)
     out = gpu_run(dl, z, k, workloads.GATE_SIGMOID_NORM, grad_scale=2.0)
-    monkeypatch.delenv("DOLOSS_LOSS_KERNEL")
+    monkeypatch.setenv("DOLOSS_LOSS_KERNEL", "alu")
     ref = gpu_run(dl, z, k, workloads.GATE_SIGMOID_NORM, grad_scale=2.0)
+    monkeypatch.delenv("DOLOSS_LOSS_KERNEL")
     for name in ("bits", "counts", "D", "origin_do"):
         assert torch.equal(getattr(out, name), getattr(ref, name)), name
     for l in range(L):
         if T <= 8192:
             assert_layer(out, l, z[l].numpy(), k, workloads.GATE_SIGMOID_NORM, grad_scale=2.0)
+            assert_layer(ref, l, z[l].numpy(), k, workloads.GATE_SIGMOID_NORM, grad_scale=2.0)
         assert float(out.loss[l]) == pytest.approx(float(ref.loss[l]), rel=1e-5)
         err = (out.dlogits[l] - ref.dlogits[l]).abs().max() / ref.dlogits[l].abs().max()
         assert float(err) <= 1e-5

@@ -42,12 +42,24 @@ def test_static_scratch_matches_workspace_path(dl, T, E, k, L, gate):
             assert float(err) <= GRAD_TOL
 
 
+def largest_static_T(dl, E, k, L=1):
+    lo, hi = 1, 1 << 24
+    while lo < hi:
+        mid = (lo + hi + 1) // 2
+        if dl.workspace_size(mid, E, k, L) <= (16 << 20):
+            lo = mid
+        else:
+            hi = mid - 1
+    return lo
+
+
 def test_static_scratch_rejects_oversized_problems(dl):
-    T, E, k = 984896 + 32, 128, 8
+    E, k = 128, 8
+    T = largest_static_T(dl, E, k) + 1
+    assert 900_000 < T < 1_000_000
     assert dl.workspace_size(T, E, k, 1) > (16 << 20)
     small = torch.zeros(64, device="cuda")
     p = ctypes.c_void_p(small.data_ptr())   # never dereferenced: the size check fails first
     st = dl.lib().do_forward_backward_static(p, T, E, k, 1, 0, 1.0, p, p, p, p, None, None, None,
                                              None)
     assert st == 6, dl.status_string(st)    # DO_ERR_WORKSPACE
-    assert dl.workspace_size(984896, E, k, 1) <= (16 << 20)
