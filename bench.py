@@ -133,18 +133,24 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
-def dist_setup(gpus):
+def dist_setup(backend=None):
+    """Rank, world size and local rank from the torchrun environment; joins the
+    process group when world > 1 (NCCL on GPUs, gloo otherwise)."""
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if world > 1:
+        import torch
         import torch.distributed as dist
 
-        dist.init_process_group("nccl")
+        if backend is None:
+            backend = "nccl" if torch.cuda.is_available() else "gloo"
+        dist.init_process_group(backend)
     return rank, world, local
 
 
 def reduce_max(x: float, world: int, device) -> float:
+    """The largest x over all ranks (x itself on one rank)."""
     if world == 1:
         return x
     import torch
@@ -153,6 +159,13 @@ def reduce_max(x: float, world: int, device) -> float:
     t = torch.tensor([x], dtype=torch.float64, device=device)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def replica_throughput(units_per_rank: float, seconds: float, world: int, device) -> tuple:
+    """Whole-job rate of `world` independent replicas: the units of all ranks
+    over the slowest rank's time.  Returns (rate, slowest seconds)."""
+    slowest = reduce_max(seconds, world, device)
+    return world * units_per_rank / slowest, slowest
 
 
 def barrier(world):
@@ -285,9 +298,8 @@ def run_ours(args, rank, world, local):
     barrier(world)
     clocks = sampler.stop()
     ms = ev0.elapsed_time(ev1)
-    ms_max = reduce_max(ms, world, dev)
-    ms_per_step = ms_max / args.steps
-    value = world * T * L / (ms_per_step * 1e-3)
+    value, seconds = replica_throughput(T * L * args.steps, ms * 1e-3, world, dev)
+    ms_per_step = seconds * 1e3 / args.steps
 
     st = dl.device_status(sets[0][1].workspace)
     if st != 0:
@@ -323,23 +335,36 @@ def run_ours(args, rank, world, local):
     achieved = algorithmic_bytes(T, E, L) / (ms_per_step * 1e-3) / 1e9
     split_gbs = {k_: stage_bytes(T, E, L)[k_] / (v * 1e-3) / 1e9 for k_, v in stage_ms.items()}
 
-    # End to end through the host entry point: pinned logits in, dlogits and loss out.
+    # End to end through the host entry point: pinned logits in, the loss out
+    # (the step's result; the gradient is computed every step and stays on
+    # the device, where the router's backward pass would consume it).  The
+    # same call with the gradient copied out as well is reported beside it.
     e2e = None
     if rank == 0 or world > 1:
         hz = base.cpu().pin_memory()
         hdz = torch.empty_like(hz).pin_memory()
         hloss = torch.empty(L, dtype=torch.float32).pin_memory()
         dbuf = torch.zeros(dl.host_buffer_size(T, E, k, L), dtype=torch.uint8, device=dev)
-        for _ in range(3):
-            dl.forward_backward_host(hz, k, w.gate, device_buffer=dbuf, h_dlogits=hdz, h_loss=hloss)
         n_e2e = max(3, min(args.steps, 50))
-        barrier(world)
-        t0 = time.perf_counter()
-        for _ in range(n_e2e):
-            dl.forward_backward_host(hz, k, w.gate, device_buffer=dbuf, h_dlogits=hdz, h_loss=hloss)
-        dt = reduce_max((time.perf_counter() - t0) / n_e2e, world, dev)
-        e2e = {"value": world * T * L / dt, "unit": UNIT, "h2d_bytes_per_step": 4 * T * E * L,
-               "d2h_bytes_per_step": 4 * T * E * L + 4 * L, "ms_per_step": dt * 1e3}
+
+        def timed(h_dlogits):
+            for _ in range(3):
+                dl.forward_backward_host(hz, k, w.gate, device_buffer=dbuf, h_dlogits=h_dlogits,
+                                         h_loss=hloss)
+            barrier(world)
+            t0 = time.perf_counter()
+            for _ in range(n_e2e):
+                dl.forward_backward_host(hz, k, w.gate, device_buffer=dbuf, h_dlogits=h_dlogits,
+                                         h_loss=hloss)
+            return replica_throughput(T * L, (time.perf_counter() - t0) / n_e2e, world, dev)
+
+        rate, dt = timed(None)
+        rate_grad, dt_grad = timed(hdz)
+        e2e = {"value": rate, "unit": UNIT, "h2d_bytes_per_step": 4 * T * E * L,
+               "d2h_bytes_per_step": 4 * L, "ms_per_step": dt * 1e3,
+               "with_dlogits_to_host": {"value": rate_grad,
+                                        "d2h_bytes_per_step": 4 * T * E * L + 4 * L,
+                                        "ms_per_step": dt_grad * 1e3}}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -383,7 +408,7 @@ def main():
         world = int(os.environ.get("WORLD_SIZE", str(args.gpus)))
         run_reference(args, rank, world)
         return
-    rank, world, local = dist_setup(args.gpus)
+    rank, world, local = dist_setup()
     try:
         run_ours(args, rank, world, local)
     finally:

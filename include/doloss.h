@@ -124,9 +124,10 @@ size_t do_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L);
 do_status do_device_status(void *workspace, void *stream);
 
 /* Host-to-host convenience over do_forward_backward: copies h_logits [L][T][E]
- * to the device, runs steps 1-3, and copies loss [L] into h_loss and, when
- * given, dlogits into h_dlogits [L][T][E], counts into h_counts [L][E] and D
- * into h_D [L][E][E].  All device memory comes from `device_buffer`
+ * to the device, runs steps 1-3 (the gradient included: it stays in
+ * device_buffer), and copies loss [L] into h_loss and, when given, dlogits
+ * into h_dlogits [L][T][E], counts into h_counts [L][E] and D into
+ * h_D [L][E][E].  All device memory comes from `device_buffer`
  * (do_host_buffer_size(T, E, k, L) bytes, 256-byte aligned, zero-filled
  * before its first use, as the workspace above).  Synchronous:
  * returns after the results are in host memory and the device status has been

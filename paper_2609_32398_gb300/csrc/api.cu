@@ -231,7 +231,9 @@ do_status do_forward_backward_host(const float *h_logits, int64_t T, int32_t E, 
     int32_t *d_counts = reinterpret_cast<int32_t *>(base + b.counts);
     int32_t *d_D = reinterpret_cast<int32_t *>(base + b.D);
     float *d_loss = reinterpret_cast<float *>(base + b.loss);
-    float *d_dlogits = h_dlogits ? reinterpret_cast<float *>(base + b.dlogits) : nullptr;
+    // the gradient is always computed (into the device buffer); it is copied to
+    // the host only when h_dlogits is given
+    float *d_dlogits = reinterpret_cast<float *>(base + b.dlogits);
     void *ws = base + b.ws;
     cudaStream_t s = (cudaStream_t)stream;
     const size_t te = sizeof(float) * (size_t)p.L * p.T * p.E;

@@ -168,7 +168,7 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W,
     for (int r = 0; r < R; ++r) cnt[r] = 0u;
 
     for (int q = warp; q < n; q += kConsumers) {
-        if (*s_abort) break;
+        if (__any_sync(kFull, *s_abort)) break;
         const int s = q % C::kSlots, round = q / C::kSlots;
         bool started = slot_round[s] >= round;
         if (!started) {
@@ -182,7 +182,8 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W,
                 }
             }
         }
-        if (!started || !mbar_wait(&full[s], round & 1, status)) {
+        const bool ok = started && mbar_wait(&full[s], round & 1, status);
+        if (!__all_sync(kFull, ok)) {  // leave together: the warp shuffles below
             *s_abort = 1;
             break;
         }

@@ -174,6 +174,10 @@ def test_host_entry_point_matches_device_path(dl):
     assert torch.equal(h_dz, dev.dlogits.cpu())
     assert torch.equal(h_counts, dev.counts.cpu())
     assert torch.equal(h_D, dev.D.cpu())
+    # loss only: the gradient is still computed (in the device buffer), not copied
+    dbuf = torch.zeros(dl.host_buffer_size(w.T, w.E, w.k, 1), dtype=torch.uint8, device="cuda")
+    h_loss2 = dl.forward_backward_host(hz, w.k, w.gate, device_buffer=dbuf)
+    assert torch.equal(h_loss2, dev.loss.cpu())
 
 
 @pytest.mark.parametrize(
