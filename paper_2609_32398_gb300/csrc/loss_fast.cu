@@ -119,6 +119,7 @@ loss_fast_kernel(const LossArgs a) {
     const int64_t t_end = min64(T, t_begin + a.tokens_per_cta);
     const int64_t stride = (int64_t)kLossFastWarps * TPW;
 
+    pdl_trigger();  // the next kernel may be scheduled (it waits for this one to finish)
     if (threadIdx.x == 0) {
         mbar_init(&bar, 1);
         fence_barrier_init();

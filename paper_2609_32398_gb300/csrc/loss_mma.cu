@@ -156,6 +156,7 @@ loss_mma_kernel(const __grid_constant__ CUtensorMap zmap, const __grid_constant_
     const int te = min(ntiles_layer, tb + a.tiles_per_cta);
     const int nt = te > tb ? te - tb : 0;
 
+    pdl_trigger();  // the next kernel may be scheduled (it waits for this one to finish)
     if (threadIdx.x == 0) {
         for (int i = 0; i < 2; ++i) {
             mbar_init(&mma_done[i], 1);

@@ -103,6 +103,10 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W,
     int *s_rowoff = reinterpret_cast<int *>(s_cooc + C::kCoocWords);
 
     pdl_trigger();
+    // Launched as a programmatic dependent of whatever ran before on the
+    // stream: wait for it before touching memory (it may have written the
+    // logits, or still read the accumulators cleared below).
+    pdl_wait();
 #pragma unroll
     for (int z = 0; z < 3; ++z)
         for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < zero.n[z];
@@ -340,9 +344,17 @@ cudaError_t run_fast(const CUtensorMap &map, const Problem &p, uint32_t *bits, i
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    dim3 grid((unsigned)sig_fast_ctas_per_problem(p), (unsigned)p.L);
-    kern<<<grid, kFastThreads, C::kSmem, s>>>(map, p.T, p.W, bits, counts, idx, cooc, zero, status);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)sig_fast_ctas_per_problem(p), (unsigned)p.L);
+    cfg.blockDim = dim3(kFastThreads);
+    cfg.dynamicSmemBytes = C::kSmem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, map, p.T, p.W, bits, counts, idx, cooc, zero, status);
 }
 
 template <int E, bool kCounts, bool kCooc>
