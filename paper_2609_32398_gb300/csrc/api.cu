@@ -53,7 +53,7 @@ HostBufLayout host_layout(const Problem &p) {
     b.bits = off;   off = round_up(off + sizeof(uint32_t) * (size_t)p.L * p.E * p.W, 256);
     b.counts = off; off = round_up(off + sizeof(int32_t) * (size_t)p.L * p.E, 256);
     b.D = off;      off = round_up(off + sizeof(int32_t) * (size_t)p.L * p.E * p.E, 256);
-    b.loss = off;   off = round_up(off + sizeof(float) * (size_t)p.L, 256);
+    b.loss = off;   off = round_up(off + sizeof(float) * (size_t)p.L + sizeof(int), 256);  // + status
     b.dlogits = off; off = round_up(off + sizeof(float) * te, 256);
     b.ws = off;     off = round_up(off + dol::workspace_bytes(p), 256);
     b.total = off;
@@ -119,7 +119,7 @@ do_status do_loss_fwd_bwd(const float *logits, const uint32_t *bits, const int32
             e = dol::launch_loss_fast(logits, idx, D, nullptr, nullptr, p, gate, d_scale,
                                       grad_scale, loss, reinterpret_cast<long long *>(origin_do),
                                       dlogits, reinterpret_cast<double *>(ws + w.partials), done,
-                                      reinterpret_cast<int *>(ws), s);
+                                      reinterpret_cast<int *>(ws), nullptr, s);
         return from_cuda(e);
     }
     return from_cuda(dol::launch_loss(logits, bits, D, p, gate, d_scale, grad_scale, loss,
@@ -127,10 +127,19 @@ do_status do_loss_fwd_bwd(const float *logits, const uint32_t *bits, const int32
                                       workspace, s));
 }
 
-do_status do_forward_backward(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
-                              int32_t gate, float grad_scale, uint32_t *bits, int32_t *counts,
-                              int32_t *D, float *loss, int64_t *origin_do, float *dlogits,
-                              void *workspace, size_t workspace_bytes, void *stream) {
+}  // extern "C"
+
+namespace {
+
+// Steps 1-3.  status_out (may be null): on the fused fast path the last loss
+// CTA ORs the device status word of this call into it (so that one copy
+// returns the loss and the status); *status_done tells whether it did.
+do_status forward_backward_impl(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
+                                int32_t gate, float grad_scale, uint32_t *bits, int32_t *counts,
+                                int32_t *D, float *loss, int64_t *origin_do, float *dlogits,
+                                void *workspace, size_t workspace_bytes, void *stream,
+                                int *status_out, bool *status_done) {
+    if (status_done) *status_done = false;
     Problem p;
     do_status st = check_sizes(T, E, k, L, &p);
     if (st != DO_OK) return st;
@@ -154,9 +163,11 @@ do_status do_forward_backward(const float *logits, int64_t T, int32_t E, int32_t
         uint8_t *idx = reinterpret_cast<uint8_t *>(ws + w.idx);
         uint32_t *parts = reinterpret_cast<uint32_t *>(ws + w.cooc_parts);
         int *n_acc = reinterpret_cast<int *>(ws + w.n_acc);
-        // origin_do is summed by the reduction kernel (integer atomics): zero it first
-        const dol::ZeroSpans zero = {{done, reinterpret_cast<int *>(origin_do), nullptr},
-                                     {(int64_t)p.L, origin_do ? 2 * (int64_t)p.L : 0, 0}};
+        // origin_do is summed by the reduction kernel (integer atomics) and
+        // status_out ORed by the loss kernel: zero them first
+        const dol::ZeroSpans zero = {{done, reinterpret_cast<int *>(origin_do), status_out},
+                                     {(int64_t)p.L, origin_do ? 2 * (int64_t)p.L : 0,
+                                      status_out ? 1 : 0}};
         int *status = reinterpret_cast<int *>(ws);
         // D <= T here (one window of tokens): the two-piece fp16 split of the
         // tensor-core path is exact when R < 2^23 (checked by loss_mma_supported)
@@ -172,13 +183,14 @@ do_status do_forward_backward(const float *logits, int64_t T, int32_t E, int32_t
             if (mma)
                 e = dol::launch_loss_mma(logits, idx, bimg, n_acc, p, 1.0f, grad_scale, loss, dlogits,
                                          reinterpret_cast<double *>(ws + w.partials), done, status,
-                                         s);
+                                         status_out, s);
             else
                 e = dol::launch_loss_fast(logits, idx, D, counts, n_acc, p, gate, 1.0f, grad_scale,
                                           loss, nullptr, dlogits,
                                           reinterpret_cast<double *>(ws + w.partials), done,
-                                          status, s);
+                                          status, status_out, s);
         }
+        if (e == cudaSuccess && status_done) *status_done = status_out != nullptr;
         return from_cuda(e);
     }
     cudaError_t e = dol::launch_signatures(logits, p, bits, counts, s);
@@ -187,6 +199,19 @@ do_status do_forward_backward(const float *logits, int64_t T, int32_t E, int32_t
         e = dol::launch_loss(logits, bits, D, p, gate, 1.0f, grad_scale, loss,
                              reinterpret_cast<long long *>(origin_do), dlogits, workspace, s);
     return from_cuda(e);
+}
+
+}  // namespace
+
+extern "C" {
+
+do_status do_forward_backward(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
+                              int32_t gate, float grad_scale, uint32_t *bits, int32_t *counts,
+                              int32_t *D, float *loss, int64_t *origin_do, float *dlogits,
+                              void *workspace, size_t workspace_bytes, void *stream) {
+    return forward_backward_impl(logits, T, E, k, L, gate, grad_scale, bits, counts, D, loss,
+                                 origin_do, dlogits, workspace, workspace_bytes, stream, nullptr,
+                                 nullptr);
 }
 
 size_t do_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L) {
@@ -238,13 +263,37 @@ do_status do_forward_backward_host(const float *h_logits, int64_t T, int32_t E, 
     cudaStream_t s = (cudaStream_t)stream;
     const size_t te = sizeof(float) * (size_t)p.L * p.T * p.E;
 
-    // A cleared status word, so that do_device_status below sees this call only.
+    // A cleared status word, so that the check below sees this call only.
     cudaError_t e = cudaMemsetAsync(ws, 0, sizeof(int), s);
     if (e == cudaSuccess) e = cudaMemcpyAsync(d_logits, h_logits, te, cudaMemcpyHostToDevice, s);
     if (e != cudaSuccess) return DO_ERR_CUDA;
-    st = do_forward_backward(d_logits, T, E, k, L, gate, grad_scale, d_bits, d_counts, d_D, d_loss,
-                             nullptr, d_dlogits, ws, dol::workspace_bytes(p), stream);
+    // the status word of this call lands right after the loss (fused path)
+    int *d_status = reinterpret_cast<int *>(d_loss + p.L);
+    bool status_done = false;
+    st = forward_backward_impl(d_logits, T, E, k, L, gate, grad_scale, d_bits, d_counts, d_D,
+                               d_loss, nullptr, d_dlogits, ws, dol::workspace_bytes(p), stream,
+                               d_status, &status_done);
     if (st != DO_OK) return st;
+    if (status_done && !h_dlogits && !h_counts && !h_D) {
+        // one copy: the loss and the status word behind it
+        struct {
+            float v[64];
+            int pad;
+        } small;
+        const size_t n = sizeof(float) * p.L + sizeof(int);
+        if (p.L <= 63) {
+            e = cudaMemcpyAsync(&small, d_loss, n, cudaMemcpyDeviceToHost, s);
+            if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+            if (e != cudaSuccess) return DO_ERR_CUDA;
+            std::memcpy(h_loss, small.v, sizeof(float) * p.L);
+            int flags = 0;
+            std::memcpy(&flags, reinterpret_cast<const char *>(&small) + sizeof(float) * p.L,
+                        sizeof(int));
+            if (flags & dol::kDevTimeout) return DO_ERR_TIMEOUT;
+            if (flags & dol::kDevOverflow) return DO_ERR_OVERFLOW;
+            return DO_OK;
+        }
+    }
     e = cudaMemcpyAsync(h_loss, d_loss, sizeof(float) * p.L, cudaMemcpyDeviceToHost, s);
     if (e == cudaSuccess && h_dlogits)
         e = cudaMemcpyAsync(h_dlogits, d_dlogits, te, cudaMemcpyDeviceToHost, s);

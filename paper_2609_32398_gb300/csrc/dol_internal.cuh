@@ -86,12 +86,12 @@ int loss_mma_ctas_per_problem(const Problem &p);
 cudaError_t launch_loss_mma(const float *logits, const uint8_t *idx, const unsigned char *bimg,
                             int *n_zero, const Problem &p, float d_scale, float grad_scale,
                             float *loss, float *dlogits, double *partials, int *done, int *status,
-                            cudaStream_t s);
+                            int *status_out, cudaStream_t s);
 cudaError_t launch_loss_fast(const float *logits, const uint8_t *idx, const int *D,
                              const int *counts, int *n_zero, const Problem &p, int gate,
                              float d_scale, float grad_scale, float *loss, long long *origin_do,
                              float *dlogits, double *partials, int *done, int *status,
-                             cudaStream_t s);
+                             int *status_out, cudaStream_t s);
 
 // Co-occurrence counts c_ab (a <= b) of one CTA are kept as a triangle whose
 // row a holds columns (a & ~3) .. E-1, so that every row starts 16-byte

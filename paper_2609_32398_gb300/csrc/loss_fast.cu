@@ -92,6 +92,7 @@ struct LossArgs {
     float *loss;
     long long *origin_do;
     int *status;
+    int *status_out;  // may be null: the last CTA ORs the status word into it
 };
 
 template <int E, int K, int kGate, bool kRFromCounts>
@@ -297,6 +298,7 @@ loss_fast_kernel(const LossArgs a) {
         if (lane == 0) {
             a.loss[layer] = (float)(sum * a.scale);
             a.done[layer] = 0;
+            if (a.status_out) atomicOr(a.status_out, *reinterpret_cast<volatile int *>(a.status));
         }
     }
     if (a.origin_do) {
@@ -469,7 +471,7 @@ cudaError_t launch_loss_fast(const float *logits, const uint8_t *idx, const int 
                              const int *counts, int *n_zero, const Problem &p, int gate,
                              float d_scale, float grad_scale, float *loss, long long *origin_do,
                              float *dlogits, double *partials, int *done, int *status,
-                             cudaStream_t s) {
+                             int *status_out, cudaStream_t s) {
     int P = 1, tpc = 32;
     loss_fast_grid(p, &P, &tpc);
     const double norm = 1.0 / ((double)p.T * (double)p.T * (double)p.k);
@@ -490,6 +492,7 @@ cudaError_t launch_loss_fast(const float *logits, const uint8_t *idx, const int 
     args.loss = loss;
     args.origin_do = origin_do;
     args.status = status;
+    args.status_out = status_out;
     if (counts) {
         if (p.E == 32) return dispatch_loss_k<32, true>(args, gate, P, p, s);
         if (p.E == 64) return dispatch_loss_k<64, true>(args, gate, P, p, s);

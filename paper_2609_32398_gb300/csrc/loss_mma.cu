@@ -109,6 +109,7 @@ struct MmaArgs {
     int *done;
     float *loss;
     int *status;
+    int *status_out;  // may be null: the last CTA ORs the status word into it
 };
 
 template <int K>
@@ -475,6 +476,7 @@ loss_mma_kernel(const __grid_constant__ CUtensorMap zmap, const __grid_constant_
         if (lane == 0) {
             a.loss[layer] = (float)(sum * a.scale);
             a.done[layer] = 0;
+            if (a.status_out) atomicOr(a.status_out, *reinterpret_cast<volatile int *>(a.status));
         }
     }
 }
@@ -531,7 +533,8 @@ int loss_mma_ctas_per_problem(const Problem &p) {
 
 cudaError_t launch_loss_mma(const float *logits, const uint8_t *idx, const unsigned char *bimg, int *n_zero, const Problem &p, float d_scale,
                             float grad_scale, float *loss, float *dlogits,
-                            double *partials, int *done, int *status, cudaStream_t s) {
+                            double *partials, int *done, int *status, int *status_out,
+                            cudaStream_t s) {
     if (!bimg) return cudaErrorInvalidValue;
     CUtensorMap zmap, dzmap;
     if (!encode_tensor_map_3d_f32(&zmap, logits, (uint64_t)p.L, (uint64_t)p.T, (uint64_t)kE, 32) ||
@@ -553,6 +556,7 @@ cudaError_t launch_loss_mma(const float *logits, const uint8_t *idx, const unsig
     args.done = done;
     args.loss = loss;
     args.status = status;
+    args.status_out = status_out;
     switch (p.k) {
         case 1: return run_mma<1>(zmap, dzmap, args, gx, p.L, s);
         case 2: return run_mma<2>(zmap, dzmap, args, gx, p.L, s);
