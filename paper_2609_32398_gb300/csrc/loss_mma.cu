@@ -452,16 +452,20 @@ loss_mma_kernel(const __grid_constant__ CUtensorMap zmap, const __grid_constant_
     tc_fence_after();
     if (warp == 0) tmem_dealloc(tmem, kTmemCols);
 
-    // CTA partial in a fixed order: a shuffle tree per warp, then the warp sums
-    double tok = (double)tok_sum;
+    // CTA partial in a fixed order: a shuffle tree per warp, then over the
+    // warp sums (fp32: at most a few hundred tokens per CTA, pairwise; the
+    // CTA partials are added in fp64)
+    float tok = tok_sum;
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) tok += __shfl_xor_sync(kFull, tok, off);
-    if (lane == 0) s_part[warp] = tok;
+    float *s_partf = reinterpret_cast<float *>(s_part);
+    if (lane == 0) s_partf[warp] = tok;
     __syncthreads();
     if (warp == 0) {
-        double v = lane < kWarps ? s_part[lane] : 0.0;
+        float vf = lane < kWarps ? s_partf[lane] : 0.0f;
 #pragma unroll
-        for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(kFull, v, off);
+        for (int off = 16; off > 0; off >>= 1) vf += __shfl_xor_sync(kFull, vf, off);
+        const double v = (double)vf;
         if (lane == 0) {
             a.partials[(int64_t)layer * gridDim.x + blockIdx.x] = v;
             // release: the partial is visible to the CTA that sees the last count

@@ -103,16 +103,6 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W,
     int *s_rowoff = reinterpret_cast<int *>(s_cooc + C::kCoocWords);
 
     pdl_trigger();
-    // Launched as a programmatic dependent of whatever ran before on the
-    // stream: wait for it before touching memory (it may have written the
-    // logits, or still read the accumulators cleared below).
-    pdl_wait();
-#pragma unroll
-    for (int z = 0; z < 3; ++z)
-        for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < zero.n[z];
-             i += (int64_t)gridDim.x * blockDim.x)
-            zero.p[z][i] = 0;
-
     // this CTA: layer blockIdx.y, a contiguous range of its 32-token tiles
     const int64_t layer = blockIdx.y;
     const int64_t per = (W + gridDim.x - 1) / gridDim.x;
@@ -120,11 +110,12 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W,
     const int64_t te = min64(W, tb + per);
     const int n = te > tb ? (int)(te - tb) : 0;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // Shared-memory set-up first: it touches no global memory, so it overlaps
+    // the end of the previous kernel on the stream.
     if (kCooc) {
         for (int i = threadIdx.x; i < C::kCoocWords; i += blockDim.x) s_cooc[i] = 0u;
         for (int a = threadIdx.x; a < E; a += blockDim.x) s_rowoff[a] = cooc_row_offset<E>(a) - (a & ~3);
     }
-
     if (threadIdx.x == 0) {
         for (int s = 0; s < C::kSlots; ++s) {
             mbar_init(&full[s], 1);
@@ -134,11 +125,20 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W,
         *s_abort = 0;
         fence_barrier_init();
     }
+    if (warp == kConsumers && lane == 0) prefetch_tensormap(&tmap);
     __syncthreads();
+    // Launched as a programmatic dependent of whatever ran before on the
+    // stream: wait for it before touching global memory (it may have written
+    // the logits, or still read the accumulators cleared below).
+    pdl_wait();
+#pragma unroll
+    for (int z = 0; z < 3; ++z)
+        for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < zero.n[z];
+             i += (int64_t)gridDim.x * blockDim.x)
+            zero.p[z][i] = 0;
 
     if (warp == kConsumers) {  // producer
         if (lane == 0 && n > 0) {
-            prefetch_tensormap(&tmap);
             int issued = 0;
             for (int q = 0; q < n; ++q) {
                 const int s = q % C::kSlots, round = q / C::kSlots;
