@@ -34,11 +34,13 @@ cooc_reduce_kernel(const uint32_t *__restrict__ partials, int P1, const int *__r
                    long long *__restrict__ origin_do, long long r_base, int r_mult) {
     constexpr int kWords = cooc_row_offset<E>(E);
     __shared__ uint32_t s_sum[kRedWarps][33];
+    __shared__ int s_n[E];  // the counts n_a, read once per CTA while the partials load
     const int e = threadIdx.x & 31, wp = threadIdx.x >> 5;
     const int word = blockIdx.x * 32 + e;
     const int layer = blockIdx.y;
     pdl_wait();
     pdl_trigger();
+    if ((int)threadIdx.x < E) s_n[threadIdx.x] = n_acc[(size_t)layer * E + threadIdx.x];
     uint32_t acc[4] = {0u, 0u, 0u, 0u};
     if (word < kWords) {
         const uint32_t *base = partials + (size_t)layer * P1 * kWords + word;
@@ -67,7 +69,6 @@ cooc_reduce_kernel(const uint32_t *__restrict__ partials, int P1, const int *__r
         }
         const int a = lo;
         const int b = (a & ~3) + (word - cooc_row_offset<E>(a));
-        const int *nl = n_acc + (size_t)layer * E;
         int *Dl = D + (size_t)layer * E * E;
         unsigned char *img = (E == 128 && bimg) ? bimg + (size_t)layer * kBImageBytes : nullptr;
         if (b < a) {
@@ -78,7 +79,7 @@ cooc_reduce_kernel(const uint32_t *__restrict__ partials, int P1, const int *__r
             // R_a = (E - 2k) n_a + T k (every row of the co-occurrence sums to k n_a)
             if (img) put_pieces(img, a, a, true, (int)(r_base + (long long)r_mult * (long long)c));
         } else {
-            const int d = nl[a] + nl[b] - 2 * (int)c;
+            const int d = s_n[a] + s_n[b] - 2 * (int)c;
             Dl[a * E + b] = d;
             Dl[b * E + a] = d;
             if (img) {
