@@ -168,6 +168,14 @@ do_status do_forward_backward_static(const float *logits, int64_t T, int32_t E, 
                                      int32_t *counts, int32_t *D, float *loss, int64_t *origin_do,
                                      float *dlogits, int32_t *status_flags, void *stream);
 
+/* Self-test of the failure path shared by every device wait: launches one
+ * thread that waits on an mbarrier which nothing completes.  Its bounded wait
+ * gives up after about one second and records the time-out in the status word
+ * of `workspace` (do_workspace_size bytes, as for the other entry points), so
+ * that do_device_status then returns DO_ERR_TIMEOUT; nothing traps or faults
+ * and the context stays usable.  Asynchronous on `stream`. */
+do_status do_selftest_wait_limit(void *workspace, void *stream);
+
 /* A static description of a status code. */
 const char *do_status_string(int32_t status);
 

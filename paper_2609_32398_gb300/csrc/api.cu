@@ -7,12 +7,20 @@
 #include <cstdlib>
 #include <cstring>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "dol_internal.cuh"
 #include "doloss.h"
 
 namespace {
 
 using dol::Problem;
+
+// An NVTX range around each entry point (a no-op unless a profiler attaches).
+struct NvtxRange {
+    explicit NvtxRange(const char *name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+};
 
 bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
@@ -66,6 +74,7 @@ extern "C" {
 
 do_status do_signatures(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
                         uint32_t *bits, int32_t *counts, void *stream) {
+    NvtxRange nvtx("do_signatures");
     Problem p;
     do_status st = check_sizes(T, E, k, L, &p);
     if (st != DO_OK) return st;
@@ -85,6 +94,7 @@ do_status do_signatures(const float *logits, int64_t T, int32_t E, int32_t k, in
 
 do_status do_pairwise_hamming(const uint32_t *bits, int64_t T, int32_t E, int32_t L, int32_t *D,
                               void *stream) {
+    NvtxRange nvtx("do_pairwise_hamming");
     Problem p;
     do_status st = check_sizes(T, E, 1, L, &p);
     if (st != DO_OK) return st;
@@ -97,6 +107,7 @@ do_status do_loss_fwd_bwd(const float *logits, const uint32_t *bits, const int32
                           int32_t E, int32_t k, int32_t L, int32_t gate, float d_scale,
                           float grad_scale, float *loss, int64_t *origin_do, float *dlogits,
                           void *workspace, size_t workspace_bytes, void *stream) {
+    NvtxRange nvtx("do_loss_fwd_bwd");
     Problem p;
     do_status st = check_sizes(T, E, k, L, &p);
     if (st != DO_OK) return st;
@@ -209,6 +220,7 @@ do_status do_forward_backward(const float *logits, int64_t T, int32_t E, int32_t
                               int32_t gate, float grad_scale, uint32_t *bits, int32_t *counts,
                               int32_t *D, float *loss, int64_t *origin_do, float *dlogits,
                               void *workspace, size_t workspace_bytes, void *stream) {
+    NvtxRange nvtx("do_forward_backward");
     return forward_backward_impl(logits, T, E, k, L, gate, grad_scale, bits, counts, D, loss,
                                  origin_do, dlogits, workspace, workspace_bytes, stream, nullptr,
                                  nullptr);
@@ -243,6 +255,7 @@ do_status do_forward_backward_host(const float *h_logits, int64_t T, int32_t E, 
                                    int32_t L, int32_t gate, float grad_scale, float *h_loss,
                                    float *h_dlogits, int32_t *h_counts, int32_t *h_D,
                                    void *device_buffer, size_t device_buffer_bytes, void *stream) {
+    NvtxRange nvtx("do_forward_backward_host");
     Problem p;
     do_status st = check_sizes(T, E, k, L, &p);
     if (st != DO_OK) return st;

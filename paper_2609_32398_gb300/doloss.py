@@ -35,6 +35,7 @@ EXPORTS = {
                                   "p", "p", "sz", "p"], "i32"),
     "do_host_buffer_size": (["i64", "i32", "i32", "i32"], "sz"),
     "do_status_string": (["i32"], "str"),
+    "do_selftest_wait_limit": (["p", "p"], "i32"),
     "do_forward_backward_static": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p", "p",
                                     "p", "p", "p", "p", "p"], "i32"),
 }
@@ -231,3 +232,10 @@ def forward_backward_static(logits, k, out: Buffers, gate=GATE_SIGMOID_NORM, gra
         out.D.data_ptr(), out.loss.data_ptr(), out.origin_do.data_ptr(), _ptr(out.dlogits),
         _ptr(status_flags), _stream(z)))
     return out
+
+
+def selftest_wait_limit(workspace: torch.Tensor) -> None:
+    """Launches the bounded-wait self-test on the current stream (see
+    include/doloss.h); do_device_status afterwards reports the time-out."""
+    _check("do_selftest_wait_limit",
+           lib().do_selftest_wait_limit(workspace.data_ptr(), _stream(workspace)))

@@ -74,3 +74,4 @@ def test_invalid_arguments_are_rejected_before_launch(dl):
                                    None, 0, None) == WS
     assert lib.do_forward_backward_host(None, 64, 8, 2, 1, 0, 1.0, fake, None, None, None, fake,
                                         1 << 30, None) == INV
+    assert lib.do_selftest_wait_limit(None, None) == WS

@@ -266,3 +266,18 @@ def test_tcgen05_and_alu_loss_kernels_agree(dl, monkeypatch, T, k, L):
         assert float(out.loss[l]) == pytest.approx(float(ref.loss[l]), rel=1e-5)
         err = (out.dlogits[l] - ref.dlogits[l]).abs().max() / ref.dlogits[l].abs().max()
         assert float(err) <= 1e-5
+
+
+def test_bounded_wait_reports_timeout_and_context_survives(dl):
+    """A device wait that nothing completes gives up, reports DO_ERR_TIMEOUT and
+    leaves the context usable (no trap, no fault, no hang)."""
+    w = workloads.get("c2", T=2048)
+    z = workloads.logits(w).cuda()
+    out = dl.Buffers(1, w.T, w.E, w.k, "cuda")
+    dl.selftest_wait_limit(out.workspace)
+    assert dl.device_status(out.workspace) == 4          # DO_ERR_TIMEOUT
+    assert dl.device_status(out.workspace) == 0          # cleared after reading
+    dl.forward_backward(z, w.k, w.gate, out=out)
+    assert dl.device_status(out.workspace) == 0
+    ref = oracle.forward_backward(z[0].cpu().numpy(), w.k, w.gate)
+    assert np.array_equal(out.D[0].cpu().numpy(), ref["D"])
