@@ -239,3 +239,34 @@ def selftest_wait_limit(workspace: torch.Tensor) -> None:
     include/doloss.h); do_device_status afterwards reports the time-out."""
     _check("do_selftest_wait_limit",
            lib().do_selftest_wait_limit(workspace.data_ptr(), _stream(workspace)))
+
+
+def all_reduce_distances(D: torch.Tensor, group=None):
+    """Sums the local Hamming matrices of the data-parallel ranks in place and
+    returns (D, d_scale), d_scale = 1 / (number of ranks): the summed matrix
+    G^g = d_scale * sum_r D_r of Global-DO (Sec. 3.1.4, Eq. global_do).  D is
+    int32 (the sum of per-rank distances stays exact); one rank or no
+    initialised process group leaves D as it is with d_scale = 1."""
+    import torch.distributed as dist
+
+    if not (dist.is_available() and dist.is_initialized()):
+        return D, 1.0
+    world = dist.get_world_size(group)
+    if world > 1:
+        dist.all_reduce(D, op=dist.ReduceOp.SUM, group=group)
+    return D, 1.0 / world
+
+
+def global_forward_backward(logits, k, gate=GATE_SIGMOID_NORM, grad_scale=1.0, group=None):
+    """Global-DO on the local tokens of this rank: signatures and the local
+    Hamming matrix, its sum over the ranks of `group`, then the loss and the
+    gradient with d_scale = 1/ranks (m stays the local token count).
+    Returns (loss [L], dlogits [L,T,E], D_global [L,E,E] int32, counts [L,E])."""
+    z = _as3d(logits)
+    L, T, E = z.shape
+    bits, counts = signatures(z, k)
+    D = pairwise_hamming(bits, T)
+    D, d_scale = all_reduce_distances(D, group)
+    loss, _, dz = loss_fwd_bwd(z, bits, D, k, gate, d_scale=d_scale, grad_scale=grad_scale,
+                               with_origin=False)
+    return loss, dz, D, counts

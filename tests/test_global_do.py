@@ -1,0 +1,89 @@
+"""Global-DO (Sec. 3.1.4, Eq. global_do): the Hamming matrices of the data-parallel
+ranks are summed and scaled by 1/ranks before the loss.
+
+CPU: two gloo ranks each hold half of the tokens; their oracle matrices, summed
+by the binding's collective helper, equal the oracle matrix of all the tokens
+(distances add over token shards) with d_scale = 1/2, and each rank's loss with
+the summed matrix matches the oracle's loss of its shard under that matrix.
+GPU: with one rank the helper reduces to the local path."""
+import os
+import socket
+import sys
+
+import numpy as np
+import pytest
+import torch
+import torch.multiprocessing as mp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, out):
+    os.environ.update({"MASTER_ADDR": "127.0.0.1", "MASTER_PORT": str(port), "RANK": str(rank),
+                       "WORLD_SIZE": str(world)})
+    sys.path.insert(0, ROOT)
+    import torch.distributed as dist
+
+    import oracle
+    from paper_2609_32398_gb300 import doloss, workloads
+
+    dist.init_process_group("gloo")
+    w = workloads.get("c2", T=2048)
+    z = workloads.logits(w)[0].numpy()
+    shard = z[rank * 1024:(rank + 1) * 1024]
+    f = oracle.select(shard, w.k)
+    D_local = torch.from_numpy(oracle.hamming(f).astype(np.int32))
+    D_sum, d_scale = doloss.all_reduce_distances(D_local.clone())
+    C = oracle.direction(shard, f, w.gate)
+    loss = oracle.loss(D_sum.numpy(), C, shard.shape[0], w.k, d_scale)
+    out[rank] = (D_sum.numpy(), d_scale, loss)
+    dist.destroy_process_group()
+
+
+def test_two_ranks_sum_distances_on_cpu():
+    import oracle
+    from paper_2609_32398_gb300 import workloads
+
+    ctx = mp.get_context("spawn")
+    manager = ctx.Manager()
+    out = manager.dict()
+    port = _free_port()
+    procs = [ctx.Process(target=_rank_main, args=(r, 2, port, out)) for r in range(2)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(timeout=180)
+    assert all(p.exitcode == 0 for p in procs)
+    w = workloads.get("c2", T=2048)
+    z = workloads.logits(w)[0].numpy()
+    D_all = oracle.hamming(oracle.select(z, w.k))
+    for r in range(2):
+        D_sum, d_scale, loss = out[r]
+        assert np.array_equal(D_sum, D_all)
+        assert d_scale == 0.5
+        shard = z[r * 1024:(r + 1) * 1024]
+        f = oracle.select(shard, w.k)
+        ref = oracle.loss(D_all, oracle.direction(shard, f, w.gate), 1024, w.k, 0.5)
+        assert loss == pytest.approx(ref, rel=1e-12)
+
+
+@pytest.mark.gpu
+def test_single_rank_global_do_equals_local_path():
+    import paper_2609_32398_gb300.doloss as dl
+    from paper_2609_32398_gb300 import workloads
+
+    w = workloads.get("c2", T=4096)
+    z = workloads.logits(w).cuda()
+    loss, dz, D, counts = dl.global_forward_backward(z, w.k, w.gate, grad_scale=2.0)
+    ref = dl.forward_backward(z, w.k, w.gate, grad_scale=2.0)
+    torch.cuda.synchronize()
+    assert torch.equal(D, ref.D) and torch.equal(counts, ref.counts)
+    assert float(loss[0]) == pytest.approx(float(ref.loss[0]), rel=1e-5)
+    err = (dz - ref.dlogits).abs().max() / ref.dlogits.abs().max()
+    assert float(err) <= 1e-5
