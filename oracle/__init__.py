@@ -64,6 +64,8 @@ def _load():
             "oracle_gate_backward": ([P, P, I64, I64, I32, I32, D, P], None),
             "oracle_origin_do": ([P, I32], I64),
             "oracle_forward_backward": ([P, I64, I32, I32, I32, D, D, P, P, P, P, P, P], ctypes.c_int),
+            "oracle_route": ([P, I64, I32, I32, I32, P, P], None),
+            "oracle_dispatch": ([P, I64, I32, I32, P, P, P], None),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -195,3 +197,26 @@ def forward_backward(z, k, gate_kind=GATE_SIGMOID_NORM, d_scale=1.0, grad_scale=
     if rc != 0:
         raise MemoryError("oracle_forward_backward ran out of host memory")
     return dict(bits=bits, counts=n, D=D, loss=lossv.value, origin_do=odo.value, dz=dz)
+
+
+def route(z, k, gate_kind=GATE_SIGMOID_NORM):
+    """Chosen experts ids [T,k] int32 (selection order) and their re-normalized
+    weights combine [T,k] float64 (Sec. 3.1.1)."""
+    z, pz = _c(z, np.float32)
+    T, E = z.shape
+    ids = np.empty((T, k), np.int32)
+    comb = np.empty((T, k), np.float64)
+    _load().oracle_route(pz, T, E, k, gate_kind, ids.ctypes.data, comb.ctypes.data)
+    return ids, comb
+
+
+def dispatch(ids, E):
+    """Expert-grouped order of the (token, choice) pairs: offsets [E+1],
+    rows [T*k] (token of each row), pos [T,k] (row of each pair)."""
+    ids, pi = _c(ids, np.int32)
+    T, k = ids.shape
+    offsets = np.empty(E + 1, np.int32)
+    rows = np.empty(T * k, np.int32)
+    pos = np.empty((T, k), np.int32)
+    _load().oracle_dispatch(pi, T, E, k, offsets.ctypes.data, rows.ctypes.data, pos.ctypes.data)
+    return offsets, rows, pos

@@ -246,3 +246,65 @@ int oracle_forward_backward(const float *z, int64_t T, int32_t E, int32_t k, int
     free(C);
     return 0;
 }
+
+/* Routing outputs of the router (Sec. 3.1.1): of the dense p_t, only the K
+ * chosen entries keep their value, and those K are re-normalized to sum to
+ * one; they weight the chosen experts' outputs.  Per token t, ids[t][q] is the
+ * q-th expert chosen by the argmax passes of oracle_select (largest logit
+ * first, equal logits lower index first) and
+ *     combine[t][q] = p_{ids[t][q],t} / sum_{q'} p_{ids[t][q'],t},
+ * with p from gate_row.  ids and combine are [T][k]. */
+void oracle_route(const float *z, int64_t T, int32_t E, int32_t k, int32_t gate, int32_t *ids,
+                  double *combine)
+{
+    double *p = (double *)malloc(sizeof(double) * (size_t)E);
+    uint8_t *taken = (uint8_t *)malloc((size_t)E);
+    for (int64_t t = 0; t < T; ++t) {
+        const float *zt = z + t * (int64_t)E;
+        int32_t *it = ids + t * (int64_t)k;
+        double *ct = combine + t * (int64_t)k;
+        for (int32_t i = 0; i < E; ++i) taken[i] = 0;
+        for (int32_t pass = 0; pass < k; ++pass) {
+            int32_t best = -1;
+            double bv = 0.0;
+            for (int32_t i = 0; i < E; ++i) {
+                if (taken[i]) continue;
+                double v = (double)zt[i];
+                if (best < 0 || v > bv) { best = i; bv = v; }
+            }
+            taken[best] = 1;
+            it[pass] = best;
+        }
+        gate_row(zt, E, gate, p);
+        double kept = 0.0;
+        for (int32_t q = 0; q < k; ++q) kept += p[it[q]];
+        for (int32_t q = 0; q < k; ++q) ct[q] = p[it[q]] / kept;
+    }
+    free(p);
+    free(taken);
+}
+
+/* Dispatch order of the routed (token, choice) pairs: grouped by expert,
+ * expert 0 first, and by token inside an expert (a stable counting sort of
+ * the pairs, taken in token order, by expert id).
+ *   offsets [E+1]: rows of expert e are offsets[e] .. offsets[e+1]-1
+ *                  (offsets[e+1] - offsets[e] = n_e, offsets[E] = T k)
+ *   rows [T k]:    the token of each row
+ *   pos [T][k]:    the row of the pair (t, q); rows[pos[t][q]] = t        */
+void oracle_dispatch(const int32_t *ids, int64_t T, int32_t E, int32_t k, int32_t *offsets,
+                     int32_t *rows, int32_t *pos)
+{
+    int64_t *fill = (int64_t *)calloc((size_t)E, sizeof(int64_t));
+    for (int32_t e = 0; e <= E; ++e) offsets[e] = 0;
+    for (int64_t t = 0; t < T; ++t)
+        for (int32_t q = 0; q < k; ++q) offsets[ids[t * k + q] + 1] += 1;
+    for (int32_t e = 0; e < E; ++e) offsets[e + 1] += offsets[e];
+    for (int64_t t = 0; t < T; ++t)
+        for (int32_t q = 0; q < k; ++q) {
+            int32_t e = ids[t * k + q];
+            int64_t r = offsets[e] + fill[e]++;
+            rows[r] = (int32_t)t;
+            pos[t * k + q] = (int32_t)r;
+        }
+    free(fill);
+}
