@@ -114,6 +114,52 @@ do_status do_forward_backward(const float *logits, int64_t T, int32_t E, int32_t
                               int32_t *D, float *loss, int64_t *origin_do, float *dlogits,
                               void *workspace, size_t workspace_bytes, void *stream);
 
+/* Routing outputs of the router (Sec. 3.1.1: of a token's normalized
+ * probabilities only the K chosen ones are kept, re-normalized to sum to
+ * one; they weigh the chosen experts' outputs), from the selection of step 1:
+ *   expert_ids     [L][T][k] int32, the chosen experts of each token in
+ *                  selection order (largest logit first, equal logits lower
+ *                  index first)
+ *   combine        [L][T][k] fp32, w_tq = p_{e_q,t} / sum_q' p_{e_q',t}
+ *                  (sigmoid-norm: s_e / sum of the chosen s; softmax: the
+ *                  softmax of the chosen logits)
+ *   counts         [L][E] int32, n_e (as do_signatures)
+ *   expert_offsets [L][E+1] int32, offsets[e] = n_0 + ... + n_{e-1},
+ *                  offsets[E] = T k
+ *   dispatch_rows  [L][T*k] int32, the routed (token, choice) pairs grouped
+ *                  by expert in expert order, tokens ascending inside an
+ *                  expert: row r holds its token id
+ *   dispatch_pos   [L][T][k] int32, the row of the pair (t, q), so that
+ *                  dispatch_rows[pos] = t
+ * expert_ids, combine and counts are required; each dispatch array may be
+ * NULL.  All are exact integers except combine, which is fp32 (a few ulp of
+ * the exact ratio); all are identical run to run.  Needs T k <= INT32_MAX
+ * (DO_ERR_UNSUPPORTED otherwise).  16-byte aligned logits, expert_ids and
+ * combine with E in {32, 64, 128} and k in {1, 2, 4, 8} take the fast
+ * selection kernel.  workspace: do_routing_workspace_size(T, E, k, L) bytes
+ * of device memory, 256-byte aligned, zero-filled before its first use (it
+ * holds the device status word, read by do_device_status, and the
+ * signatures).  Asynchronous on `stream`. */
+do_status do_routing(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L, int32_t gate,
+                     int32_t *expert_ids, float *combine, int32_t *counts,
+                     int32_t *expert_offsets, int32_t *dispatch_rows, int32_t *dispatch_pos,
+                     void *workspace, size_t workspace_bytes, void *stream);
+
+size_t do_routing_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L);
+
+/* do_forward_backward that also writes the routing outputs of do_routing
+ * (expert_ids, combine required; expert_offsets, dispatch_rows, dispatch_pos
+ * may each be NULL) from the same selection pass over the logits, so the
+ * logits are read once for both the loss and the dispatch.  Same workspace
+ * as do_forward_backward. */
+do_status do_forward_backward_routed(const float *logits, int64_t T, int32_t E, int32_t k,
+                                     int32_t L, int32_t gate, float grad_scale, uint32_t *bits,
+                                     int32_t *counts, int32_t *D, float *loss, int64_t *origin_do,
+                                     float *dlogits, int32_t *expert_ids, float *combine,
+                                     int32_t *expert_offsets, int32_t *dispatch_rows,
+                                     int32_t *dispatch_pos, void *workspace,
+                                     size_t workspace_bytes, void *stream);
+
 /* Device workspace, in bytes, that do_loss_fwd_bwd and do_forward_backward
  * need for these sizes (0 if the sizes are invalid). */
 size_t do_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L);

@@ -53,6 +53,35 @@ struct HostBufLayout {
     size_t logits, bits, counts, D, loss, dlogits, ws, total;
 };
 
+// Routing outputs of one call (Sec. 3.1.1): ids and combine are required,
+// the dispatch arrays may each be null.
+struct RouteArgs {
+    int32_t *ids;
+    float *combine;
+    int32_t *offsets, *rows, *pos;
+};
+
+// Checks shared by the entry points that write routing outputs: the row and
+// token indices of the dispatch arrays are int32.
+do_status check_route(const Problem &p, const RouteArgs &r) {
+    if ((int64_t)p.T * p.k > (int64_t)INT_MAX) return DO_ERR_UNSUPPORTED;
+    if (!r.ids || !r.combine) return DO_ERR_INVALID_ARG;
+    if (!aligned(r.ids, 4) || !aligned(r.combine, 4) || (r.offsets && !aligned(r.offsets, 4)) ||
+        (r.rows && !aligned(r.rows, 4)) || (r.pos && !aligned(r.pos, 4)))
+        return DO_ERR_INVALID_ARG;
+    return DO_OK;
+}
+
+// The vector stores of the fast selection kernel want 16-byte aligned rows.
+bool route_fast_ok(const RouteArgs *r) {
+    return !r || (aligned(r->ids, 16) && aligned(r->combine, 16));
+}
+
+// Workspace of do_routing: [status word | pad to 256 B | signatures [L][E][W]].
+size_t routing_ws_bytes(const Problem &p) {
+    return dol::kWsHeader + round_up(sizeof(uint32_t) * (size_t)p.L * p.E * p.W, 256);
+}
+
 HostBufLayout host_layout(const Problem &p) {
     HostBufLayout b;
     size_t off = 0;
@@ -149,7 +178,8 @@ do_status forward_backward_impl(const float *logits, int64_t T, int32_t E, int32
                                 int32_t gate, float grad_scale, uint32_t *bits, int32_t *counts,
                                 int32_t *D, float *loss, int64_t *origin_do, float *dlogits,
                                 void *workspace, size_t workspace_bytes, void *stream,
-                                int *status_out, bool *status_done) {
+                                int *status_out, bool *status_done,
+                                const RouteArgs *ra = nullptr) {
     if (status_done) *status_done = false;
     Problem p;
     do_status st = check_sizes(T, E, k, L, &p);
@@ -161,11 +191,13 @@ do_status forward_backward_impl(const float *logits, int64_t T, int32_t E, int32
         !aligned(loss, 4) || (dlogits && !aligned(dlogits, 4)) ||
         (origin_do && !aligned(origin_do, 8)))
         return DO_ERR_INVALID_ARG;
+    if (ra && (st = check_route(p, *ra)) != DO_OK) return st;
     if (!workspace || !aligned(workspace, 256) || workspace_bytes < dol::workspace_bytes(p))
         return DO_ERR_WORKSPACE;
     cudaStream_t s = (cudaStream_t)stream;
+    const dol::RouteOut route = {ra ? ra->ids : nullptr, ra ? ra->combine : nullptr, gate};
     if (dol::signatures_fast_supported(logits, p) && dol::loss_fast_supported(p, logits, D, dlogits) &&
-        aligned(bits, 16)) {
+        aligned(bits, 16) && route_fast_ok(ra)) {
         // signatures (+ per-CTA co-occurrence counts) -> reduction to C -> loss,
         // which builds D = n_i + n_j - 2 c_ij and writes D and the counts
         const dol::WsLayout w = dol::ws_layout(p);
@@ -186,7 +218,9 @@ do_status forward_backward_impl(const float *logits, int64_t T, int32_t E, int32
                          dol::loss_mma_supported(p, gate, logits, D, dlogits);
         unsigned char *bimg = mma ? reinterpret_cast<unsigned char *>(ws + w.bimg) : nullptr;
         cudaError_t e =
-            dol::launch_signatures_fast(logits, p, bits, n_acc, idx, parts, zero, status, s);
+            ra ? dol::launch_signatures_fast_routed(logits, p, bits, n_acc, idx, parts, zero, status,
+                                                    route, s)
+               : dol::launch_signatures_fast(logits, p, bits, n_acc, idx, parts, zero, status, s);
         if (e == cudaSuccess)
             e = dol::launch_cooc_reduce(parts, dol::sig_fast_ctas_per_problem(p), n_acc, p, D,
                                         counts, bimg, reinterpret_cast<long long *>(origin_do), s);
@@ -201,14 +235,20 @@ do_status forward_backward_impl(const float *logits, int64_t T, int32_t E, int32
                                           reinterpret_cast<double *>(ws + w.partials), done,
                                           status, status_out, s);
         }
+        // the dispatch order needs the final counts: after the loss kernel
+        if (e == cudaSuccess && ra)
+            e = dol::launch_route_dispatch(bits, counts, ra->ids, p, ra->offsets, ra->rows,
+                                           ra->pos, s);
         if (e == cudaSuccess && status_done) *status_done = status_out != nullptr;
         return from_cuda(e);
     }
-    cudaError_t e = dol::launch_signatures(logits, p, bits, counts, s);
+    cudaError_t e = dol::launch_signatures(logits, p, bits, counts, s, route);
     if (e == cudaSuccess) e = dol::launch_hamming(bits, p, D, s);
     if (e == cudaSuccess)
         e = dol::launch_loss(logits, bits, D, p, gate, 1.0f, grad_scale, loss,
                              reinterpret_cast<long long *>(origin_do), dlogits, workspace, s);
+    if (e == cudaSuccess && ra)
+        e = dol::launch_route_dispatch(bits, counts, ra->ids, p, ra->offsets, ra->rows, ra->pos, s);
     return from_cuda(e);
 }
 
@@ -224,6 +264,60 @@ do_status do_forward_backward(const float *logits, int64_t T, int32_t E, int32_t
     return forward_backward_impl(logits, T, E, k, L, gate, grad_scale, bits, counts, D, loss,
                                  origin_do, dlogits, workspace, workspace_bytes, stream, nullptr,
                                  nullptr);
+}
+
+do_status do_forward_backward_routed(const float *logits, int64_t T, int32_t E, int32_t k,
+                                     int32_t L, int32_t gate, float grad_scale, uint32_t *bits,
+                                     int32_t *counts, int32_t *D, float *loss, int64_t *origin_do,
+                                     float *dlogits, int32_t *expert_ids, float *combine,
+                                     int32_t *expert_offsets, int32_t *dispatch_rows,
+                                     int32_t *dispatch_pos, void *workspace,
+                                     size_t workspace_bytes, void *stream) {
+    NvtxRange nvtx("do_forward_backward_routed");
+    const RouteArgs ra = {expert_ids, combine, expert_offsets, dispatch_rows, dispatch_pos};
+    return forward_backward_impl(logits, T, E, k, L, gate, grad_scale, bits, counts, D, loss,
+                                 origin_do, dlogits, workspace, workspace_bytes, stream, nullptr,
+                                 nullptr, &ra);
+}
+
+do_status do_routing(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L, int32_t gate,
+                     int32_t *expert_ids, float *combine, int32_t *counts,
+                     int32_t *expert_offsets, int32_t *dispatch_rows, int32_t *dispatch_pos,
+                     void *workspace, size_t workspace_bytes, void *stream) {
+    NvtxRange nvtx("do_routing");
+    Problem p;
+    do_status st = check_sizes(T, E, k, L, &p);
+    if (st != DO_OK) return st;
+    if (gate != DO_GATE_SIGMOID_NORM && gate != DO_GATE_SOFTMAX) return DO_ERR_INVALID_ARG;
+    const RouteArgs ra = {expert_ids, combine, expert_offsets, dispatch_rows, dispatch_pos};
+    if ((st = check_route(p, ra)) != DO_OK) return st;
+    if (!logits || !counts || !aligned(logits, 4) || !aligned(counts, 4)) return DO_ERR_INVALID_ARG;
+    if (!workspace || !aligned(workspace, 256) || workspace_bytes < routing_ws_bytes(p))
+        return DO_ERR_WORKSPACE;
+    cudaStream_t s = (cudaStream_t)stream;
+    char *ws = static_cast<char *>(workspace);
+    uint32_t *bits = reinterpret_cast<uint32_t *>(ws + dol::kWsHeader);
+    const dol::RouteOut route = {expert_ids, combine, gate};
+    cudaError_t e;
+    if (dol::signatures_fast_supported(logits, p) && route_fast_ok(&ra)) {
+        const dol::ZeroSpans none = {{nullptr, nullptr, nullptr}, {0, 0, 0}};
+        e = cudaMemsetAsync(counts, 0, sizeof(int) * (size_t)p.L * p.E, s);
+        if (e == cudaSuccess)
+            e = dol::launch_signatures_fast_routed(logits, p, bits, counts, nullptr, nullptr, none,
+                                                   reinterpret_cast<int *>(ws), route, s);
+    } else {
+        e = dol::launch_signatures(logits, p, bits, counts, s, route);
+    }
+    if (e == cudaSuccess)
+        e = dol::launch_route_dispatch(bits, counts, expert_ids, p, expert_offsets, dispatch_rows,
+                                       dispatch_pos, s);
+    return from_cuda(e);
+}
+
+size_t do_routing_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L) {
+    Problem p;
+    if (check_sizes(T, E, k, L, &p) != DO_OK) return 0;
+    return routing_ws_bytes(p);
 }
 
 size_t do_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L) {

@@ -26,6 +26,16 @@ struct Problem {
     int64_t W;    // 32-bit words per signature, ceil(T/32)
 };
 
+// Routing outputs written by the selection pass (Sec. 3.1.1); ids == nullptr
+// means none.  Both arrays are [L][T][k], one row per token, the chosen
+// experts in selection order (largest logit first, equal logits lower index
+// first) with their re-normalized weights.
+struct RouteOut {
+    int *ids;
+    float *combine;
+    int gate;  // 0 sigmoid-norm, 1 softmax
+};
+
 // Up to three int ranges that a kernel clears for the kernels after it.
 struct ZeroSpans {
     int *p[3];
@@ -56,8 +66,10 @@ inline size_t workspace_bytes(const Problem &p) { return ws_layout(p).total; }
 int loss_blocks_per_problem(const Problem &p);
 
 // Launchers (return the first CUDA error, cudaSuccess otherwise).
+// route.ids != nullptr: the routing outputs are written too.
 cudaError_t launch_signatures(const float *logits, const Problem &p, uint32_t *bits,
-                              int *counts, cudaStream_t s);
+                              int *counts, cudaStream_t s,
+                              const RouteOut &route = RouteOut{nullptr, nullptr, 0});
 cudaError_t launch_hamming(const uint32_t *bits, const Problem &p, int *D, cudaStream_t s);
 cudaError_t launch_hamming_accumulate(const uint32_t *bits, const Problem &p, int *D, int *counts,
                                       cudaStream_t s);
@@ -71,6 +83,17 @@ bool signatures_fast_supported(const float *logits, const Problem &p);
 cudaError_t launch_signatures_fast(const float *logits, const Problem &p, uint32_t *bits,
                                    int *counts, uint8_t *idx, uint32_t *cooc, const ZeroSpans &zero,
                                    int *status, cudaStream_t s);
+// The same kernel with the routing outputs (ids and combine 16-byte aligned).
+cudaError_t launch_signatures_fast_routed(const float *logits, const Problem &p, uint32_t *bits,
+                                          int *counts, uint8_t *idx, uint32_t *cooc,
+                                          const ZeroSpans &zero, int *status,
+                                          const RouteOut &route, cudaStream_t s);
+// Dispatch order of the routed (token, choice) pairs from the signatures and
+// the final counts: offsets [L][E+1], rows [L][T k], pos [L][T][k] (each may
+// be null).  Launched as a programmatic dependent of the previous kernel.
+cudaError_t launch_route_dispatch(const uint32_t *bits, const int *counts, const int *ids,
+                                  const Problem &p, int *offsets, int *rows, int *pos,
+                                  cudaStream_t s);
 bool loss_fast_supported(const Problem &p, const float *logits, const int *D, const float *dlogits);
 cudaError_t launch_idx_from_bits(const uint32_t *bits, const Problem &p, uint8_t *idx, int *zero_ptr,
                                  int zero_n, cudaStream_t s);
@@ -172,6 +195,20 @@ __device__ __forceinline__ double warp_sum_fixed(const double *x, int64_t n) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(kFull, s, o);
     return s;
+}
+
+// Weight of a chosen expert before the re-normalization over the chosen set
+// (Sec. 3.1.1), for a token whose first chosen logit (the largest) is v0:
+//   softmax        exp(v - v0)                       (= p_v / p_v0)
+//   sigmoid-norm   sigmoid(v)                        if v0 >= 0
+//                  exp(v - v0) (1 + e^v0) / (1 + e^v) if v0 < 0 (= s_v / s_v0)
+// The dense normaliser cancels in the ratio.  The two sigmoid forms are equal
+// in exact arithmetic; the second keeps every chosen weight away from
+// underflow when all chosen logits are very negative.
+__device__ __forceinline__ float route_raw_weight(float v, float v0, int gate) {
+    if (gate == 1) return expf(v - v0);
+    if (v0 >= 0.0f) return 1.0f / (1.0f + expf(-v));
+    return expf(v - v0) * ((1.0f + expf(v0)) / (1.0f + expf(v)));
 }
 
 __device__ __forceinline__ float warp_max(float v) {

@@ -3,7 +3,9 @@
 //   n_i  = ||F_i||_1            (App. C.3)
 // Top-K is taken on the raw fp32 logits; equal values go to the lower expert
 // index.  A warp owns 32 consecutive tokens, i.e. one 32-bit word of every
-// signature, so no two warps ever write the same word.
+// signature, so no two warps ever write the same word.  With routing outputs
+// the kernel also writes each token's chosen experts in selection order and
+// their weights re-normalized over the chosen set (Sec. 3.1.1).
 #include <climits>
 #include <cmath>
 
@@ -20,7 +22,7 @@ constexpr int kSigThreads = 256;
 template <int R>
 __global__ void __launch_bounds__(kSigThreads)
 sig_generic_kernel(const float *__restrict__ logits, int64_t T, int E, int k, int64_t W,
-                   uint32_t *__restrict__ bits, int *__restrict__ counts) {
+                   uint32_t *__restrict__ bits, int *__restrict__ counts, RouteOut route) {
     __shared__ int s_cnt[32 * R];
     const int layer = blockIdx.y;
     const float *z = logits + (int64_t)layer * T * E;
@@ -43,6 +45,9 @@ sig_generic_kernel(const float *__restrict__ logits, int64_t T, int E, int k, in
         const int nt = (int)min64(32, T - t0);
         for (int tt = 0; tt < nt; ++tt) {
             const float *zt = z + (t0 + tt) * E;
+            // routing outputs of this token: ids in selection order, and the
+            // chosen logits parked in combine until the weights replace them
+            const int64_t roff = ((int64_t)layer * T + t0 + tt) * k;
             float v[R];
 #pragma unroll
             for (int r = 0; r < R; ++r) {
@@ -68,6 +73,22 @@ sig_generic_kernel(const float *__restrict__ logits, int64_t T, int E, int k, in
                     if (take) { bv = ov; bi = oi; }
                 }
                 if ((bi & 31) == lane) sel |= 1u << (bi >> 5);
+                if (route.ids && lane == 0) {
+                    route.ids[roff + q] = bi;
+                    route.combine[roff + q] = bv;
+                }
+            }
+            if (route.ids) {
+                // w_q = u_q / sum u over the chosen set (u: route_raw_weight);
+                // the lane-strided sum and the butterfly fix the order
+                __syncwarp();
+                float *ct = route.combine + roff;
+                const float v0 = ct[0];
+                float part = 0.0f;
+                for (int q = lane; q < k; q += 32) part += route_raw_weight(ct[q], v0, route.gate);
+                const float sum = warp_sum(part);
+                __syncwarp();
+                for (int q = lane; q < k; q += 32) ct[q] = route_raw_weight(ct[q], v0, route.gate) / sum;
             }
 #pragma unroll
             for (int r = 0; r < R; ++r) word[r] |= ((sel >> r) & 1u) << tt;
@@ -93,30 +114,31 @@ sig_generic_kernel(const float *__restrict__ logits, int64_t T, int E, int k, in
 
 template <int R>
 cudaError_t run_generic(const float *logits, const Problem &p, uint32_t *bits, int *counts,
-                        cudaStream_t s) {
+                        const RouteOut &route, cudaStream_t s) {
     const int warps = kSigThreads / 32;
     int64_t blocks = (p.W + warps - 1) / warps;
     const int64_t cap = (p.L >= 1024) ? 1 : (2048 / p.L);
     if (blocks > cap) blocks = cap;
     if (blocks < 1) blocks = 1;
     dim3 grid((unsigned)blocks, (unsigned)p.L);
-    sig_generic_kernel<R><<<grid, kSigThreads, 0, s>>>(logits, p.T, p.E, p.k, p.W, bits, counts);
+    sig_generic_kernel<R><<<grid, kSigThreads, 0, s>>>(logits, p.T, p.E, p.k, p.W, bits, counts,
+                                                             route);
     return cudaGetLastError();
 }
 
 }  // namespace
 
 cudaError_t launch_signatures(const float *logits, const Problem &p, uint32_t *bits, int *counts,
-                              cudaStream_t s) {
+                              cudaStream_t s, const RouteOut &route) {
     cudaError_t e = cudaMemsetAsync(counts, 0, sizeof(int) * (size_t)p.L * p.E, s);
     if (e != cudaSuccess) return e;
     const int r = (p.E + 31) / 32;
-    if (r <= 1) return run_generic<1>(logits, p, bits, counts, s);
-    if (r <= 2) return run_generic<2>(logits, p, bits, counts, s);
-    if (r <= 4) return run_generic<4>(logits, p, bits, counts, s);
-    if (r <= 8) return run_generic<8>(logits, p, bits, counts, s);
-    if (r <= 16) return run_generic<16>(logits, p, bits, counts, s);
-    return run_generic<32>(logits, p, bits, counts, s);
+    if (r <= 1) return run_generic<1>(logits, p, bits, counts, route, s);
+    if (r <= 2) return run_generic<2>(logits, p, bits, counts, route, s);
+    if (r <= 4) return run_generic<4>(logits, p, bits, counts, route, s);
+    if (r <= 8) return run_generic<8>(logits, p, bits, counts, route, s);
+    if (r <= 16) return run_generic<16>(logits, p, bits, counts, route, s);
+    return run_generic<32>(logits, p, bits, counts, route, s);
 }
 
 }  // namespace dol

@@ -38,6 +38,11 @@ EXPORTS = {
     "do_selftest_wait_limit": (["p", "p"], "i32"),
     "do_forward_backward_static": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p", "p",
                                     "p", "p", "p", "p", "p"], "i32"),
+    "do_routing": (["p", "i64", "i32", "i32", "i32", "i32", "p", "p", "p", "p", "p", "p", "p", "sz",
+                    "p"], "i32"),
+    "do_routing_workspace_size": (["i64", "i32", "i32", "i32"], "sz"),
+    "do_forward_backward_routed": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p", "p",
+                                    "p", "p", "p", "p", "p", "p", "p", "p", "p", "sz", "p"], "i32"),
 }
 
 _CT = {"p": ctypes.c_void_p, "i64": ctypes.c_int64, "i32": ctypes.c_int32,
@@ -188,6 +193,68 @@ def forward_backward(logits, k, gate=GATE_SIGMOID_NORM, grad_scale=1.0, out: Buf
         out.D.data_ptr(), out.loss.data_ptr(), out.origin_do.data_ptr(), _ptr(dl),
         out.workspace.data_ptr(), out.workspace.numel(), _stream(z)))
     return out
+
+
+class Routing:
+    """Routing outputs (Sec. 3.1.1) for one shape: expert_ids [L,T,k] int32,
+    combine [L,T,k] fp32, counts [L,E] int32, offsets [L,E+1] int32,
+    rows [L,T*k] int32, pos [L,T,k] int32, and the do_routing workspace."""
+
+    def __init__(self, L, T, E, k, device="cuda", with_dispatch=True):
+        self.shape = (L, T, E, k)
+        self.expert_ids = torch.empty(L, T, k, dtype=torch.int32, device=device)
+        self.combine = torch.empty(L, T, k, dtype=torch.float32, device=device)
+        self.counts = torch.empty(L, E, dtype=torch.int32, device=device)
+        if with_dispatch:
+            self.offsets = torch.empty(L, E + 1, dtype=torch.int32, device=device)
+            self.rows = torch.empty(L, T * k, dtype=torch.int32, device=device)
+            self.pos = torch.empty(L, T, k, dtype=torch.int32, device=device)
+        else:
+            self.offsets = self.rows = self.pos = None
+        n = int(lib().do_routing_workspace_size(T, E, k, L))
+        if n == 0:
+            raise ValueError("invalid sizes")
+        self.workspace = torch.zeros(n, dtype=torch.uint8, device=device)
+
+
+def routing(logits, k, gate=GATE_SIGMOID_NORM, out: Routing | None = None):
+    """do_routing: the chosen experts, their re-normalized combine weights and
+    the expert-grouped dispatch order; returns the Routing holding them."""
+    z = _as3d(logits)
+    L, T, E = z.shape
+    if out is None:
+        out = Routing(L, T, E, k, z.device)
+    if out.shape != (L, T, E, k):
+        raise ValueError("routing buffers were made for another shape")
+    _check("do_routing", lib().do_routing(
+        z.data_ptr(), T, E, k, L, gate, out.expert_ids.data_ptr(), out.combine.data_ptr(),
+        out.counts.data_ptr(), _ptr(out.offsets), _ptr(out.rows), _ptr(out.pos),
+        out.workspace.data_ptr(), out.workspace.numel(), _stream(z)))
+    return out
+
+
+def forward_backward_routed(logits, k, gate=GATE_SIGMOID_NORM, grad_scale=1.0,
+                            out: Buffers | None = None, route: Routing | None = None,
+                            with_grad=True):
+    """do_forward_backward_routed: steps 1-3 plus the routing outputs from the
+    same selection pass.  Returns (Buffers, Routing); route.counts and
+    route.workspace are not used (the counts are out.counts)."""
+    z = _as3d(logits)
+    L, T, E = z.shape
+    if out is None:
+        out = Buffers(L, T, E, k, z.device, with_grad)
+    if route is None:
+        route = Routing(L, T, E, k, z.device)
+    if out.shape != (L, T, E, k) or route.shape != (L, T, E, k):
+        raise ValueError("output buffers were made for another shape")
+    dl = out.dlogits if with_grad else None
+    _check("do_forward_backward_routed", lib().do_forward_backward_routed(
+        z.data_ptr(), T, E, k, L, gate, grad_scale, out.bits.data_ptr(), out.counts.data_ptr(),
+        out.D.data_ptr(), out.loss.data_ptr(), out.origin_do.data_ptr(), _ptr(dl),
+        route.expert_ids.data_ptr(), route.combine.data_ptr(), _ptr(route.offsets),
+        _ptr(route.rows), _ptr(route.pos), out.workspace.data_ptr(), out.workspace.numel(),
+        _stream(z)))
+    return out, route
 
 
 def device_status(workspace: torch.Tensor) -> int:

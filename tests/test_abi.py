@@ -75,3 +75,35 @@ def test_invalid_arguments_are_rejected_before_launch(dl):
     assert lib.do_forward_backward_host(None, 64, 8, 2, 1, 0, 1.0, fake, None, None, None, fake,
                                         1 << 30, None) == INV
     assert lib.do_selftest_wait_limit(None, None) == WS
+
+
+def test_routing_entry_points_validate_on_the_host(dl):
+    lib = dl.lib()
+    fake = ctypes.c_void_p(0x10000)
+    odd = ctypes.c_void_p(0x10002)
+    INV, UNS, WS = 1, 2, 6
+    big_ws = 1 << 30
+    assert dl.lib().do_routing_workspace_size(0, 8, 2, 1) == 0
+    # status word + padding + the signatures [L][E][W]
+    assert dl.lib().do_routing_workspace_size(1000, 8, 2, 3) == 256 + 4 * 3 * 8 * 32
+    assert lib.do_routing(fake, 64, 8, 2, 1, 0, None, fake, fake, None, None, None, fake, big_ws,
+                          None) == INV                                        # no expert_ids
+    assert lib.do_routing(fake, 64, 8, 2, 1, 0, fake, None, fake, None, None, None, fake, big_ws,
+                          None) == INV                                        # no combine
+    assert lib.do_routing(fake, 64, 8, 2, 1, 0, fake, fake, None, None, None, None, fake, big_ws,
+                          None) == INV                                        # no counts
+    assert lib.do_routing(fake, 64, 8, 2, 1, 2, fake, fake, fake, None, None, None, fake, big_ws,
+                          None) == INV                                        # bad gate
+    assert lib.do_routing(fake, 64, 8, 2, 1, 0, fake, fake, fake, odd, None, None, fake, big_ws,
+                          None) == INV                                        # misaligned offsets
+    assert lib.do_routing(fake, 64, 8, 2, 1, 0, fake, fake, fake, None, None, None, fake, 16,
+                          None) == WS                                         # small workspace
+    # (E - 1) T fits int32 but T k does not: dispatch rows are int32
+    assert lib.do_routing(fake, (1 << 30) + 1, 2, 2, 1, 0, fake, fake, fake, None, None, None, fake,
+                          big_ws, None) == UNS
+    assert lib.do_forward_backward_routed(fake, 64, 8, 2, 1, 0, 1.0, fake, fake, fake, fake, None,
+                                          None, None, fake, None, None, None, fake, big_ws,
+                                          None) == INV                        # no expert_ids
+    assert lib.do_forward_backward_routed(fake, 64, 8, 2, 1, 0, 1.0, fake, fake, fake, fake, None,
+                                          None, fake, fake, None, None, None, fake, 8,
+                                          None) == WS
