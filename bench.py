@@ -56,6 +56,13 @@ def stage_bytes(T, E, L=1):
     }
 
 
+def routing_bytes(T, E, k, L=1):
+    """Bytes the routing outputs must move once: logits read (4TE), expert ids,
+    combine weights, dispatch rows and positions written (4Tk each), counts
+    and offsets (4E + 4(E+1)) -- per problem."""
+    return L * (4 * T * E + 16 * T * k + 8 * E + 4)
+
+
 def measured_peaks():
     try:
         return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
@@ -264,12 +271,27 @@ def run_ours(args, rank, world, local):
 
     warm = max(3, args.warmup)
     if args.quick:
-        # profiling mode: a few plain steps, nothing else (used under ncu)
+        # profiling mode: a few plain calls of one entry point, nothing else
+        # (used under ncu)
+        if args.quick_path == "loss":
+            call, ws = step, sets[0][1].workspace
+        else:
+            route = dl.Routing(L, T, E, k, dev)
+            if args.quick_path == "routing":
+                def call(i):
+                    dl.routing(sets[i % N_SETS][0], k, w.gate, out=route)
+                ws = route.workspace
+            else:
+                def call(i):
+                    dl.forward_backward_routed(sets[i % N_SETS][0], k, w.gate, 1.0,
+                                               out=sets[i % N_SETS][1], route=route)
+                ws = sets[0][1].workspace
         for i in range(warm + args.steps):
-            step(i)
+            call(i)
         torch.cuda.synchronize()
-        st = dl.device_status(sets[0][1].workspace)
-        print(json.dumps({"quick": True, "steps": warm + args.steps, "status": st}), flush=True)
+        st = dl.device_status(ws)
+        print(json.dumps({"quick": True, "path": args.quick_path, "steps": warm + args.steps,
+                          "status": st}), flush=True)
         return
     sampler = ClockSampler(local)
     sampler.start()
@@ -326,6 +348,35 @@ def run_ours(args, rank, world, local):
         stage_ms["signatures"] += e[0].elapsed_time(e[1]) / reps
         stage_ms["pairwise_hamming"] += e[1].elapsed_time(e[2]) / reps
         stage_ms["loss_fwd_bwd"] += e[2].elapsed_time(e[3]) / reps
+    # Routing outputs (Sec. 3.1.1): do_routing alone, and the DO-loss step that
+    # also writes them from the same selection pass.
+    routes = [dl.Routing(L, T, E, k, dev) for _ in range(N_SETS)]
+    for r in range(2 * N_SETS):
+        dl.routing(sets[r % N_SETS][0], k, w.gate, out=routes[r % N_SETS])
+        dl.forward_backward_routed(sets[r % N_SETS][0], k, w.gate, 1.0, out=sets[r % N_SETS][1],
+                                   route=routes[r % N_SETS])
+    torch.cuda.synchronize()
+
+    def time_calls(fn):
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for r in range(reps):
+            fn(r)
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / reps
+
+    route_ms = time_calls(lambda r: dl.routing(sets[r % N_SETS][0], k, w.gate, out=routes[r % N_SETS]))
+    routed_ms = time_calls(lambda r: dl.forward_backward_routed(
+        sets[r % N_SETS][0], k, w.gate, 1.0, out=sets[r % N_SETS][1], route=routes[r % N_SETS]))
+    plain_ms = time_calls(lambda r: dl.forward_backward(sets[r % N_SETS][0], k, w.gate, 1.0,
+                                                        out=sets[r % N_SETS][1]))
+    for r in range(N_SETS):
+        for ws in (routes[r].workspace, sets[r][1].workspace):
+            st = dl.device_status(ws)
+            if st != 0:
+                raise RuntimeError(f"device status after the routing runs: {dl.status_string(st)}")
     peaks = measured_peaks()
     peak = peaks["hbm_gbs"] if peaks else 6800.0
     peak_src = "of measured" if peaks else "of fallback"
@@ -387,6 +438,20 @@ def run_ours(args, rank, world, local):
                          "traffic": profiled_traffic("do_forward_backward")},
             "split_entry_points": {"us": {k_: v * 1e3 for k_, v in stage_ms.items()},
                                    "GB/s": split_gbs},
+            "routing": {
+                "entry": "do_routing (selection with ids and combine weights, dispatch order)",
+                "us_per_call": route_ms * 1e3, "tokens_per_s": T * L / (route_ms * 1e-3),
+                "roofline": {"bound": "hbm", "kernel": "do_routing",
+                             "achieved": routing_bytes(T, E, k, L) / (route_ms * 1e-3) / 1e9,
+                             "peak": peak, "unit": "GB/s",
+                             "frac": routing_bytes(T, E, k, L) / (route_ms * 1e-3) / 1e9 / peak,
+                             "peak_source": peak_src,
+                             "algorithmic_bytes": routing_bytes(T, E, k, L),
+                             "traffic": profiled_traffic("do_routing")},
+                "fused": {"entry": "do_forward_backward_routed",
+                          "us_per_call": routed_ms * 1e3,
+                          "us_per_call_without_routing": plain_ms * 1e3},
+                "reps": reps},
             "clocks": clocks, "e2e": e2e, "gpu_launches": KERNELS_PER_STEP * args.steps,
             "cpu_baseline": cpu,
         }
@@ -402,6 +467,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--quick", action="store_true",
                     help="run warmup+steps plain steps and exit (for profilers)")
+    ap.add_argument("--quick-path", choices=["loss", "routing", "routed"], default="loss",
+                    help="entry point of --quick: do_forward_backward, do_routing or "
+                         "do_forward_backward_routed")
     args = ap.parse_args()
     if args.impl == "reference":
         rank = int(os.environ.get("RANK", "0"))

@@ -77,9 +77,15 @@ bool route_fast_ok(const RouteArgs *r) {
     return !r || (aligned(r->ids, 16) && aligned(r->combine, 16));
 }
 
-// Workspace of do_routing: [status word | pad to 256 B | signatures [L][E][W]].
+// Workspace of do_routing: [status word | pad to 256 B | signatures [L][E][W] |
+// dispatch scratch [L][E][route chunks]].
+size_t routing_bits_bytes(const Problem &p) {
+    return round_up(sizeof(uint32_t) * (size_t)p.L * p.E * p.W, 256);
+}
+
 size_t routing_ws_bytes(const Problem &p) {
-    return dol::kWsHeader + round_up(sizeof(uint32_t) * (size_t)p.L * p.E * p.W, 256);
+    return dol::kWsHeader + routing_bits_bytes(p) +
+           round_up(sizeof(int) * (size_t)p.L * p.E * (size_t)dol::route_chunks(p), 256);
 }
 
 HostBufLayout host_layout(const Problem &p) {
@@ -238,7 +244,7 @@ do_status forward_backward_impl(const float *logits, int64_t T, int32_t E, int32
         // the dispatch order needs the final counts: after the loss kernel
         if (e == cudaSuccess && ra)
             e = dol::launch_route_dispatch(bits, counts, ra->ids, p, ra->offsets, ra->rows,
-                                           ra->pos, s);
+                                           ra->pos, reinterpret_cast<int *>(ws + w.route_base), s);
         if (e == cudaSuccess && status_done) *status_done = status_out != nullptr;
         return from_cuda(e);
     }
@@ -248,7 +254,9 @@ do_status forward_backward_impl(const float *logits, int64_t T, int32_t E, int32
         e = dol::launch_loss(logits, bits, D, p, gate, 1.0f, grad_scale, loss,
                              reinterpret_cast<long long *>(origin_do), dlogits, workspace, s);
     if (e == cudaSuccess && ra)
-        e = dol::launch_route_dispatch(bits, counts, ra->ids, p, ra->offsets, ra->rows, ra->pos, s);
+        e = dol::launch_route_dispatch(
+            bits, counts, ra->ids, p, ra->offsets, ra->rows, ra->pos,
+            reinterpret_cast<int *>(static_cast<char *>(workspace) + dol::ws_layout(p).route_base), s);
     return from_cuda(e);
 }
 
@@ -309,8 +317,9 @@ do_status do_routing(const float *logits, int64_t T, int32_t E, int32_t k, int32
         e = dol::launch_signatures(logits, p, bits, counts, s, route);
     }
     if (e == cudaSuccess)
-        e = dol::launch_route_dispatch(bits, counts, expert_ids, p, expert_offsets, dispatch_rows,
-                                       dispatch_pos, s);
+        e = dol::launch_route_dispatch(
+            bits, counts, expert_ids, p, expert_offsets, dispatch_rows, dispatch_pos,
+            reinterpret_cast<int *>(ws + dol::kWsHeader + routing_bits_bytes(p)), s);
     return from_cuda(e);
 }
 

@@ -51,8 +51,10 @@ struct ZeroSpans {
 //   n_acc           [L][E] int32, counts summed by the signatures CTAs (kept at
 //                   zero between calls: the loss kernel clears it after use)
 //   bimg            [L][kBImageBytes], the fp16 image of D' (E = 128 only)
+//   route_base      [L][E][route chunks] int32, scratch of the dispatch order
+//                   (inside idx when it fits there: it is used after the loss)
 struct WsLayout {
-    size_t done, partials, idx, cooc_parts, n_acc, bimg, total;
+    size_t done, partials, idx, cooc_parts, n_acc, bimg, route_base, total;
     int max_parts;  // partial slots per problem
 };
 // Signatures CTAs per problem on the fast path: min(SMs, kMaxSigCtas) / L.
@@ -90,10 +92,12 @@ cudaError_t launch_signatures_fast_routed(const float *logits, const Problem &p,
                                           const RouteOut &route, cudaStream_t s);
 // Dispatch order of the routed (token, choice) pairs from the signatures and
 // the final counts: offsets [L][E+1], rows [L][T k], pos [L][T][k] (each may
-// be null).  Launched as a programmatic dependent of the previous kernel.
+// be null).  chunk_base: scratch of route_chunks(p) * E * L ints.  Launched as
+// programmatic dependents of the previous kernel.
+int64_t route_chunks(const Problem &p);
 cudaError_t launch_route_dispatch(const uint32_t *bits, const int *counts, const int *ids,
                                   const Problem &p, int *offsets, int *rows, int *pos,
-                                  cudaStream_t s);
+                                  int *chunk_base, cudaStream_t s);
 bool loss_fast_supported(const Problem &p, const float *logits, const int *D, const float *dlogits);
 cudaError_t launch_idx_from_bits(const uint32_t *bits, const Problem &p, uint8_t *idx, int *zero_ptr,
                                  int zero_n, cudaStream_t s);

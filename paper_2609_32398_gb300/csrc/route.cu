@@ -3,8 +3,8 @@
 // the chosen experts' outputs.  The selection pass that builds the signatures
 // writes the chosen experts and those weights (the kRoute instantiations of
 // the kernel in sig_fast.cuh, or the generic kernel); this file launches them
-// and holds the dispatch kernel, which puts the routed (token, choice) pairs
-// in expert order:
+// and holds the two dispatch kernels, which put the routed (token, choice)
+// pairs in expert order:
 //   offsets[e] = n_0 + ... + n_{e-1}, offsets[E] = T k
 //   rows[offsets[e] + r] = the r-th token (ascending) routed to expert e
 //   pos[t][q] = the row of the pair (t, q), so rows[pos[t][q]] = t.
@@ -16,34 +16,40 @@
 namespace dol {
 namespace {
 
-constexpr int kDispThreads = 512;
-constexpr int kDispWarps = kDispThreads / 32;
+constexpr int kScanThreads = 256;
+constexpr int kScanWarps = kScanThreads / 32;
+constexpr int kScatterThreads = 256;
+constexpr int kMaxChunkWords = 32;
+constexpr int kBatch = 8;  // independent global loads a scatter thread keeps in flight
 
-// One CTA per (expert, problem).  It sums the counts of the experts before
-// its own for the offset, then walks the expert's signature words in passes of
-// kDispThreads consecutive words: a block-wide exclusive scan of the words'
-// population counts gives every word its first row, and the word's set bits
-// (its tokens, ascending) take the rows after it.
-__global__ void __launch_bounds__(kDispThreads)
-route_dispatch_kernel(const uint32_t *__restrict__ bits, const int *__restrict__ counts,
-                      const int *__restrict__ ids, int64_t T, int E, int k, int64_t W,
-                      int *__restrict__ offsets, int *__restrict__ rows, int *__restrict__ pos) {
-    __shared__ int s_warp[kDispWarps];
+// Kernel 1, one CTA per (expert e, problem): the offset of e (the counts of
+// the experts before it) and, for every chunk of C = route_chunk_words(p)
+// signature words, the first row of e's tokens in that chunk:
+//   chunk_base[c] = offsets[e] + (set bits of F_e in chunks 0 .. c-1).
+// A thread sums its chunk's population counts; a block-wide exclusive scan
+// over the chunks of a pass (kScanThreads chunks) and the running total of
+// the passes before it give the bases.
+__global__ void __launch_bounds__(kScanThreads)
+route_scan_kernel(const uint32_t *__restrict__ bits, const int *__restrict__ counts, int E,
+                  int64_t W, int C, int64_t nchunks, int *__restrict__ offsets,
+                  int *__restrict__ chunk_base) {
+    __shared__ int s_warp[kScanWarps];
     __shared__ int s_base;
     const int e = blockIdx.x, layer = blockIdx.y;
     const int tid = threadIdx.x, lane = tid & 31, wp = tid >> 5;
-    // the signatures, counts and ids come from the kernels before this one
+    // the signatures and counts come from the kernels before this one
     pdl_wait();
+    pdl_trigger();
     const int *cl = counts + (size_t)layer * E;
     int part = 0;
-    for (int i = tid; i < e; i += kDispThreads) part += cl[i];
+    for (int i = tid; i < e; i += kScanThreads) part += cl[i];
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(kFull, part, o);
     if (lane == 0) s_warp[wp] = part;
     __syncthreads();
     if (tid == 0) {
         int b = 0;
-        for (int q = 0; q < kDispWarps; ++q) b += s_warp[q];
+        for (int q = 0; q < kScanWarps; ++q) b += s_warp[q];
         s_base = b;
         if (offsets) {
             offsets[(size_t)layer * (E + 1) + e] = b;
@@ -51,18 +57,24 @@ route_dispatch_kernel(const uint32_t *__restrict__ bits, const int *__restrict__
         }
     }
     __syncthreads();
-    if (!rows && !pos) return;
-    const int64_t Tk = T * k;
-    int run = s_base;  // first row of this pass
+    if (!chunk_base) return;
+    int run = s_base;
     const uint32_t *be = bits + ((size_t)layer * E + e) * W;
-    const int *il = ids + (size_t)layer * T * k;
-    int *rl = rows ? rows + (size_t)layer * T * k : nullptr;
-    int *pl = pos ? pos + (size_t)layer * T * k : nullptr;
-    for (int64_t w0 = 0; w0 < W; w0 += kDispThreads) {
-        const int64_t w = w0 + tid;
-        uint32_t b = w < W ? __ldg(be + w) : 0u;
-        const int c = __popc(b);
-        int x = c;  // inclusive scan inside the warp
+    int *cb = chunk_base + ((size_t)layer * E + e) * nchunks;
+    for (int64_t c0 = 0; c0 < nchunks; c0 += kScanThreads) {
+        const int64_t c = c0 + tid;
+        int n = 0;
+        if (c < nchunks) {
+            // all of the chunk's loads in flight at once (C <= kMaxChunkWords)
+            const int64_t wa = c * C;
+            uint32_t v[kMaxChunkWords];
+#pragma unroll
+            for (int j = 0; j < kMaxChunkWords; ++j)
+                v[j] = (j < C && wa + j < W) ? __ldg(be + wa + j) : 0u;
+#pragma unroll
+            for (int j = 0; j < kMaxChunkWords; ++j) n += __popc(v[j]);
+        }
+        int x = n;  // inclusive scan inside the warp
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
             const int y = __shfl_up_sync(kFull, x, o);
@@ -73,33 +85,88 @@ route_dispatch_kernel(const uint32_t *__restrict__ bits, const int *__restrict__
         __syncthreads();
         int before = 0, total = 0;
 #pragma unroll
-        for (int q = 0; q < kDispWarps; ++q) {
+        for (int q = 0; q < kScanWarps; ++q) {
             const int v = s_warp[q];
             before += q < wp ? v : 0;
             total += v;
         }
-        int r = run + before + x - c;
-        while (b) {
-            const int bit = __ffs(b) - 1;
-            b &= b - 1;
-            const int64_t t = 32 * w + bit;
-            // bits past T are zero and the rows of expert e end at offsets[e+1]
-            // when the signatures and counts come from one complete selection;
-            // after an aborted one (a timed-out wait, reported in the status
-            // word) they may not: never index outside the arrays
-            if (t >= T || r < 0 || r >= Tk) break;
-            if (rl) rl[r] = (int)t;
-            if (pl) {
-                const int *it = il + t * k;
-                for (int q = 0; q < k; ++q)
-                    if (__ldg(it + q) == e) {
-                        pl[t * k + q] = r;
-                        break;
-                    }
-            }
-            ++r;
-        }
+        if (c < nchunks) cb[c] = run + before + x - n;
         run += total;
+    }
+}
+
+// Kernel 2, one CTA per (chunk of C signature words = 32 C tokens, problem):
+// the chunk's words of every expert and their exclusive prefix counts inside
+// the chunk go to shared memory; then every routed pair (t, q) of the chunk,
+// read in order from ids, gets its row
+//   r = chunk_base[e][c] + (set bits of F_e in the chunk before t)
+// written to pos[t][q] (in order) and rows[r] = t.
+__global__ void __launch_bounds__(kScatterThreads)
+route_scatter_kernel(const uint32_t *__restrict__ bits, const int *__restrict__ ids,
+                     const int *__restrict__ chunk_base, int64_t T, int E, int k, int64_t W,
+                     int C, int64_t nchunks, int *__restrict__ rows, int *__restrict__ pos) {
+    extern __shared__ int smem_i[];
+    uint32_t *s_bits = reinterpret_cast<uint32_t *>(smem_i);  // [E][C]
+    int *s_pre = smem_i + E * C;                              // [E][C]
+    int *s_cb = s_pre + E * C;                                // [E]
+    const int64_t c = blockIdx.x;
+    const int layer = blockIdx.y;
+    const int tid = threadIdx.x;
+    pdl_wait();
+    const int64_t w0 = c * C;
+    const int nw = (int)min64(C, W - w0);
+    const uint32_t *bl = bits + (size_t)layer * E * W;
+    for (int i0 = tid; i0 < E * C; i0 += kScatterThreads * kBatch) {
+        uint32_t v[kBatch];
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+            const int i = i0 + u * kScatterThreads;
+            const int e = i / C, j = i - e * C;
+            v[u] = (i < E * C && j < nw) ? __ldg(bl + (size_t)e * W + w0 + j) : 0u;
+        }
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+            const int i = i0 + u * kScatterThreads;
+            if (i < E * C) s_bits[i] = v[u];
+        }
+    }
+    for (int e = tid; e < E; e += kScatterThreads)
+        s_cb[e] = chunk_base[((size_t)layer * E + e) * nchunks + c];
+    __syncthreads();
+    for (int e = tid; e < E; e += kScatterThreads) {
+        int acc = 0;
+        for (int j = 0; j < C; ++j) {
+            s_pre[e * C + j] = acc;
+            acc += __popc(s_bits[e * C + j]);
+        }
+    }
+    __syncthreads();
+    const int64_t Tk = T * k;
+    const int64_t i0 = 32 * w0 * k, i1 = min64(T, 32 * (w0 + nw)) * k;
+    const int *il = ids + (size_t)layer * Tk;
+    int *rl = rows ? rows + (size_t)layer * Tk : nullptr;
+    int *pl = pos ? pos + (size_t)layer * Tk : nullptr;
+    for (int64_t ib = i0 + tid; ib < i1; ib += (int64_t)kScatterThreads * kBatch) {
+        int ev[kBatch];
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+            const int64_t i = ib + (int64_t)u * kScatterThreads;
+            ev[u] = i < i1 ? __ldg(il + i) : -1;
+        }
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+            const int64_t i = ib + (int64_t)u * kScatterThreads;
+            const int e = ev[u];
+            // ids come from one complete selection; after an aborted one (a
+            // timed-out wait, reported in the status word) they may not:
+            // never index outside the arrays
+            if (i >= i1 || (unsigned)e >= (unsigned)E) continue;
+            const int64_t t = i / k;
+            const int j = (int)(t / 32 - w0), b = (int)(t & 31);
+            const int r = s_cb[e] + s_pre[e * C + j] + __popc(s_bits[e * C + j] & ((1u << b) - 1u));
+            if (pl) pl[i] = r;
+            if (rl && r >= 0 && r < Tk) rl[r] = (int)t;
+        }
     }
 }
 
@@ -117,21 +184,47 @@ cudaError_t launch_signatures_fast_routed(const float *logits, const Problem &p,
     return dispatch_mode<128, true>(map, p, bits, counts, idx, cooc, zero, status, route, s);
 }
 
+// Signature words per dispatch chunk: a power of two with about 2048 routed
+// pairs per chunk (32 C k), at most kMaxChunkWords, and the chunk's words of
+// all experts (E C) within 4096 words of shared memory.
+int route_chunk_words(const Problem &p) {
+    int lim = 64 / p.k;
+    if (lim > kMaxChunkWords) lim = kMaxChunkWords;
+    if (lim > 4096 / p.E) lim = 4096 / p.E;
+    int c = 1;
+    while (2 * c <= lim) c *= 2;
+    return c;
+}
+
+int64_t route_chunks(const Problem &p) {
+    const int C = route_chunk_words(p);
+    return (p.W + C - 1) / C;
+}
+
 cudaError_t launch_route_dispatch(const uint32_t *bits, const int *counts, const int *ids,
                                   const Problem &p, int *offsets, int *rows, int *pos,
-                                  cudaStream_t s) {
+                                  int *chunk_base, cudaStream_t s) {
     if (!offsets && !rows && !pos) return cudaSuccess;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)p.E, (unsigned)p.L);
-    cfg.blockDim = dim3(kDispThreads);
-    cfg.stream = s;
+    const int C = route_chunk_words(p);
+    const int64_t nchunks = route_chunks(p);
+    int *cb = (rows || pos) ? chunk_base : nullptr;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)p.E, (unsigned)p.L);
+    cfg.blockDim = dim3(kScanThreads);
+    cfg.stream = s;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, route_dispatch_kernel, bits, counts, ids, p.T, p.E, p.k, p.W,
-                              offsets, rows, pos);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, route_scan_kernel, bits, counts, p.E, p.W, C, nchunks,
+                                       offsets, cb);
+    if (e != cudaSuccess || !cb) return e;
+    cfg.gridDim = dim3((unsigned)nchunks, (unsigned)p.L);
+    cfg.blockDim = dim3(kScatterThreads);
+    cfg.dynamicSmemBytes = sizeof(int) * (size_t)(2 * p.E * C + p.E);
+    return cudaLaunchKernelEx(&cfg, route_scatter_kernel, bits, ids, (const int *)cb, p.T, p.E,
+                              p.k, p.W, C, nchunks, rows, pos);
 }
 
 }  // namespace dol

@@ -68,6 +68,7 @@ def run_routing(dl, z_cpu, k, gate, **kw):
     (2500, 33, 5, 2, 0, True),       # generic
     (640, 256, 8, 1, 1, False),      # generic
     (97, 16, 16, 1, 0, True),        # k = E
+    (500, 130, 100, 1, 0, True),     # one signature word per dispatch chunk
 ])
 def test_routing_matches_oracle(dl, T, E, k, L, gate, ties):
     z = workloads.random_logits(T, E, L=L, seed=T + 7 * E + k, ties=ties)
