@@ -14,11 +14,13 @@ Readings where the paper is silent:
     rank, nor twice on one rank.
   * Loads and token volumes are real numbers (the controller works on moving
     averages); tau is fixed before the loop, as Algorithm rem_allocation
-    computes it once; the floor of the second case is taken as printed.
+    computes it once, from the loads summed in rank order; the floor of the
+    second case is taken as printed.
   * Ties: the least-loaded rank with the lowest index; among equal scores the
     lowest expert index.
   * A rank is full when it holds D replicas; the loop ends when every rank is
     full or the best score of the chosen receiver is not positive.
+  * MaxVio of a batch without tokens (tau = 0) is 0.
 """
 from __future__ import annotations
 
@@ -36,9 +38,12 @@ def rank_loads(counts, expert_rank, R):
 
 
 def maxvio(loads):
-    """App. E: MaxVio = max_r |L_r / tau - 1|, tau = (1/|R|) sum_r L_r."""
+    """App. E: MaxVio = max_r |L_r / tau - 1|, tau = (1/|R|) sum_r L_r.  A batch
+    without tokens (tau = 0) has no violation: 0."""
     R = len(loads)
     tau = sum(float(x) for x in loads) / R
+    if tau == 0.0:
+        return 0.0
     return max(abs(float(x) / tau - 1.0) for x in loads)
 
 
@@ -59,7 +64,10 @@ def rem_allocate(loads, expert_tokens, expert_rank, D):
     L = [float(x) for x in loads]
     T = [float(x) for x in expert_tokens]
     R = len(L)
-    tau = sum(L) / R
+    total = 0.0
+    for x in L:                 # the loads summed in rank order
+        total += x
+    tau = total / R
     placed = [[] for _ in range(R)]        # experts replicated on each rank
     A = []
     while True:

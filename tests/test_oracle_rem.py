@@ -26,6 +26,7 @@ def test_maxvio_closed_forms():
     assert rem.maxvio([7, 7, 7, 7]) == 0.0                 # uniform
     assert rem.maxvio([0, 0, 0, 12]) == pytest.approx(3.0)  # one rank holds all: |R| - 1
     assert rem.maxvio([0, 10]) == pytest.approx(1.0)        # an idle rank counts as well
+    assert rem.maxvio([0, 0, 0]) == 0.0                      # no tokens, no violation
 
 
 def test_rank_loads_sum_the_resident_experts():
