@@ -222,6 +222,45 @@ do_status do_forward_backward_static(const float *logits, int64_t T, int32_t E, 
  * and the context stays usable.  Asynchronous on `stream`. */
 do_status do_selftest_wait_limit(void *workspace, void *stream);
 
+/* MaxVio (App. E) of each problem's counts: with expert_rank [E] (device
+ * int32) the rank that holds each expert, L_r = sum of counts[l][e] over the
+ * experts on rank r and tau = (1/R) sum_r L_r,
+ *   maxvio[l] = max_r |L_r / tau - 1|   (0 when the problem has no tokens).
+ * counts [L][E] device int32 (as written by do_signatures, do_routing or
+ * do_forward_backward); rank_loads [L][R] device int64 (may be NULL) receives
+ * L_r; maxvio [L] device double.  L_r and tau are exact (integer sums), and
+ * the result is the double-precision evaluation of the formula.  status_flags
+ * (device int32, may be NULL): bit 2 (value 4) is ORed in when an expert_rank
+ * entry lies outside [0, R) (that expert is then left out).  R <= 4096.
+ * Asynchronous on `stream`. */
+do_status do_maxvio(const int32_t *counts, const int32_t *expert_rank, int32_t E, int32_t R,
+                    int32_t L, int64_t *rank_loads, double *maxvio, int32_t *status_flags,
+                    void *stream);
+
+/* Global-batch replica allocation of the Replica Expert Mechanism (Sec. 3.2,
+ * Eq. benefit_score; App. B.1, Algorithm rem_allocation).  Host function: all
+ * pointers are host memory, and it returns when done.
+ *   loads [R]          historical rank loads L_r (e.g. moving averages of
+ *                      do_maxvio's rank_loads)
+ *   expert_tokens [E]  token volume T_e of each expert
+ *   expert_rank [E]    home rank of each expert, in [0, R)
+ *   D                  replica slots per rank
+ * tau = (1/R) sum_r L_r is fixed at the start.  Repeatedly: the receiver is
+ * the least-loaded rank with a free slot (lowest index on ties); among the
+ * experts not on it and not yet replicated there, sent from their home rank
+ * r_s, the one of largest Benefit Score S(e, r_s, r_r, tau) (lowest index on
+ * ties) is placed with Delta = S tokens, and L_r_r += Delta, L_r_s -= Delta,
+ * T_e -= Delta.  It stops when every rank is full or the best score is not
+ * positive.  Writes the placements in order to placed_expert, placed_sender,
+ * placed_receiver and placed_tokens (capacity R*D each; may be NULL when
+ * D = 0), their number to *n_placed and the updated loads to loads_out [R].
+ * DO_ERR_INVALID_ARG for an expert_rank entry outside [0, R). */
+do_status do_rem_allocate(const double *loads, const double *expert_tokens,
+                          const int32_t *expert_rank, int32_t R, int32_t E, int32_t D,
+                          int32_t *placed_expert, int32_t *placed_sender,
+                          int32_t *placed_receiver, double *placed_tokens, int32_t *n_placed,
+                          double *loads_out);
+
 /* A static description of a status code. */
 const char *do_status_string(int32_t status);
 

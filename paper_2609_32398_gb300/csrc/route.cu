@@ -23,26 +23,42 @@ constexpr int kMaxChunkWords = 32;
 constexpr int kBatch = 8;  // independent global loads a scatter thread keeps in flight
 
 // Kernel 1, one CTA per (expert e, problem): the offset of e (the counts of
-// the experts before it) and, for every chunk of C = route_chunk_words(p)
-// signature words, the first row of e's tokens in that chunk:
+// the experts before it) and, for every chunk of C = 2^lc signature words,
+// the first row of e's tokens in that chunk:
 //   chunk_base[c] = offsets[e] + (set bits of F_e in chunks 0 .. c-1).
 // A thread sums its chunk's population counts; a block-wide exclusive scan
 // over the chunks of a pass (kScanThreads chunks) and the running total of
-// the passes before it give the bases.
+// the passes before it give the bases.  The first pass's loads are issued
+// together with those of the counts, before any barrier.
 __global__ void __launch_bounds__(kScanThreads)
 route_scan_kernel(const uint32_t *__restrict__ bits, const int *__restrict__ counts, int E,
-                  int64_t W, int C, int64_t nchunks, int *__restrict__ offsets,
+                  int64_t W, int lc, int64_t nchunks, int *__restrict__ offsets,
                   int *__restrict__ chunk_base) {
     __shared__ int s_warp[kScanWarps];
     __shared__ int s_base;
     const int e = blockIdx.x, layer = blockIdx.y;
     const int tid = threadIdx.x, lane = tid & 31, wp = tid >> 5;
+    const int C = 1 << lc;
+    const uint32_t *be = bits + ((size_t)layer * E + e) * W;
+    // population count of chunk c of F_e, its loads all in flight at once
+    auto chunk_count = [&](int64_t c) {
+        uint32_t v[kMaxChunkWords];
+        const int64_t wa = c << lc;
+#pragma unroll
+        for (int j = 0; j < kMaxChunkWords; ++j)
+            v[j] = (c < nchunks && j < C && wa + j < W) ? __ldg(be + wa + j) : 0u;
+        int n = 0;
+#pragma unroll
+        for (int j = 0; j < kMaxChunkWords; ++j) n += __popc(v[j]);
+        return n;
+    };
     // the signatures and counts come from the kernels before this one
     pdl_wait();
     pdl_trigger();
     const int *cl = counts + (size_t)layer * E;
     int part = 0;
-    for (int i = tid; i < e; i += kScanThreads) part += cl[i];
+    for (int i = tid; i < e; i += kScanThreads) part += __ldg(cl + i);
+    int n = chunk_base ? chunk_count(tid) : 0;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(kFull, part, o);
     if (lane == 0) s_warp[wp] = part;
@@ -59,28 +75,17 @@ route_scan_kernel(const uint32_t *__restrict__ bits, const int *__restrict__ cou
     __syncthreads();
     if (!chunk_base) return;
     int run = s_base;
-    const uint32_t *be = bits + ((size_t)layer * E + e) * W;
     int *cb = chunk_base + ((size_t)layer * E + e) * nchunks;
     for (int64_t c0 = 0; c0 < nchunks; c0 += kScanThreads) {
         const int64_t c = c0 + tid;
-        int n = 0;
-        if (c < nchunks) {
-            // all of the chunk's loads in flight at once (C <= kMaxChunkWords)
-            const int64_t wa = c * C;
-            uint32_t v[kMaxChunkWords];
-#pragma unroll
-            for (int j = 0; j < kMaxChunkWords; ++j)
-                v[j] = (j < C && wa + j < W) ? __ldg(be + wa + j) : 0u;
-#pragma unroll
-            for (int j = 0; j < kMaxChunkWords; ++j) n += __popc(v[j]);
-        }
+        if (c0 > 0) n = chunk_count(c);
         int x = n;  // inclusive scan inside the warp
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
             const int y = __shfl_up_sync(kFull, x, o);
             if (lane >= o) x += y;
         }
-        __syncthreads();  // the previous pass has read s_warp
+        __syncthreads();  // s_warp is free again
         if (lane == 31) s_warp[wp] = x;
         __syncthreads();
         int before = 0, total = 0;
@@ -95,39 +100,56 @@ route_scan_kernel(const uint32_t *__restrict__ bits, const int *__restrict__ cou
     }
 }
 
-// Kernel 2, one CTA per (chunk of C signature words = 32 C tokens, problem):
-// the chunk's words of every expert and their exclusive prefix counts inside
-// the chunk go to shared memory; then every routed pair (t, q) of the chunk,
-// read in order from ids, gets its row
-//   r = chunk_base[e][c] + (set bits of F_e in the chunk before t)
-// written to pos[t][q] (in order) and rows[r] = t.
+// Kernel 2, one CTA per (chunk of C = 2^lc signature words = 32 C tokens,
+// problem): the chunk's words of every expert and their exclusive prefix
+// counts inside the chunk go to shared memory.  Then
+//   rows: a thread per (expert e, word) writes the word's tokens, ascending,
+//         from row chunk_base[e][c] + (set bits of F_e in the chunk before
+//         the word) on (runs of consecutive rows per expert);
+//   pos:  the routed pairs (t, q) of the chunk are read from ids in order and
+//         each gets r = chunk_base[e][c] + (set bits of F_e in the chunk
+//         before t), written to pos[t][q] in order.
+// Indices inside a problem fit int32 (T k <= INT32_MAX); lk = log2 k when k
+// is a power of two (the pair index is then split by a shift), else -1.
 __global__ void __launch_bounds__(kScatterThreads)
 route_scatter_kernel(const uint32_t *__restrict__ bits, const int *__restrict__ ids,
-                     const int *__restrict__ chunk_base, int64_t T, int E, int k, int64_t W,
-                     int C, int64_t nchunks, int *__restrict__ rows, int *__restrict__ pos) {
+                     const int *__restrict__ chunk_base, int T, int E, int k, int lk, int64_t W,
+                     int lc, int64_t nchunks, int *__restrict__ rows, int *__restrict__ pos) {
     extern __shared__ int smem_i[];
+    const int C = 1 << lc, EC = E << lc;
     uint32_t *s_bits = reinterpret_cast<uint32_t *>(smem_i);  // [E][C]
-    int *s_pre = smem_i + E * C;                              // [E][C]
-    int *s_cb = s_pre + E * C;                                // [E]
+    int *s_pre = smem_i + EC;                                 // [E][C]
+    int *s_cb = s_pre + EC;                                   // [E]
     const int64_t c = blockIdx.x;
     const int layer = blockIdx.y;
     const int tid = threadIdx.x;
     pdl_wait();
-    const int64_t w0 = c * C;
+    const int64_t w0 = c << lc;
     const int nw = (int)min64(C, W - w0);
+    const int Tk = T * k;
+    const int i0 = (int)(32 * w0) * k, i1 = (int)min64(T, 32 * (w0 + nw)) * k;
+    const int *il = ids + (size_t)layer * Tk;
+    // the first batch of this thread's expert ids: loaded before the barriers
+    // below, so that its latency overlaps the shared-memory set-up
+    int ev[kBatch];
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
+        const int i = i0 + tid + u * kScatterThreads;
+        ev[u] = (pos && i < i1) ? __ldg(il + i) : -1;
+    }
     const uint32_t *bl = bits + (size_t)layer * E * W;
-    for (int i0 = tid; i0 < E * C; i0 += kScatterThreads * kBatch) {
+    for (int m0 = tid; m0 < EC; m0 += kScatterThreads * kBatch) {
         uint32_t v[kBatch];
 #pragma unroll
         for (int u = 0; u < kBatch; ++u) {
-            const int i = i0 + u * kScatterThreads;
-            const int e = i / C, j = i - e * C;
-            v[u] = (i < E * C && j < nw) ? __ldg(bl + (size_t)e * W + w0 + j) : 0u;
+            const int i = m0 + u * kScatterThreads;
+            const int e = i >> lc, j = i & (C - 1);
+            v[u] = (i < EC && j < nw) ? __ldg(bl + (size_t)e * W + w0 + j) : 0u;
         }
 #pragma unroll
         for (int u = 0; u < kBatch; ++u) {
-            const int i = i0 + u * kScatterThreads;
-            if (i < E * C) s_bits[i] = v[u];
+            const int i = m0 + u * kScatterThreads;
+            if (i < EC) s_bits[i] = v[u];
         }
     }
     for (int e = tid; e < E; e += kScatterThreads)
@@ -136,36 +158,48 @@ route_scatter_kernel(const uint32_t *__restrict__ bits, const int *__restrict__ 
     for (int e = tid; e < E; e += kScatterThreads) {
         int acc = 0;
         for (int j = 0; j < C; ++j) {
-            s_pre[e * C + j] = acc;
-            acc += __popc(s_bits[e * C + j]);
+            s_pre[(e << lc) + j] = acc;
+            acc += __popc(s_bits[(e << lc) + j]);
         }
     }
     __syncthreads();
-    const int64_t Tk = T * k;
-    const int64_t i0 = 32 * w0 * k, i1 = min64(T, 32 * (w0 + nw)) * k;
-    const int *il = ids + (size_t)layer * Tk;
-    int *rl = rows ? rows + (size_t)layer * Tk : nullptr;
-    int *pl = pos ? pos + (size_t)layer * Tk : nullptr;
-    for (int64_t ib = i0 + tid; ib < i1; ib += (int64_t)kScatterThreads * kBatch) {
-        int ev[kBatch];
+    if (rows) {
+        int *rl = rows + (size_t)layer * Tk;
+        for (int i = tid; i < EC; i += kScatterThreads) {
+            uint32_t b = s_bits[i];
+            int r = s_cb[i >> lc] + s_pre[i];
+            const int tb = (int)(32 * (w0 + (i & (C - 1))));
+            while (b) {
+                const int bit = __ffs(b) - 1;
+                b &= b - 1;
+                // bits past T are zero and the rows of an expert end before the
+                // next expert's when the signatures and counts come from one
+                // complete selection; after an aborted one (a timed-out wait,
+                // reported in the status word) they may not: stay in bounds
+                if (r >= 0 && r < Tk) rl[r] = tb + bit;
+                ++r;
+            }
+        }
+    }
+    if (!pos) return;
+    int *pl = pos + (size_t)layer * Tk;
+    for (int ib = i0 + tid; ib < i1; ib += kScatterThreads * kBatch) {
+        if (ib != i0 + tid) {
 #pragma unroll
-        for (int u = 0; u < kBatch; ++u) {
-            const int64_t i = ib + (int64_t)u * kScatterThreads;
-            ev[u] = i < i1 ? __ldg(il + i) : -1;
+            for (int u = 0; u < kBatch; ++u) {
+                const int i = ib + u * kScatterThreads;
+                ev[u] = i < i1 ? __ldg(il + i) : -1;
+            }
         }
 #pragma unroll
         for (int u = 0; u < kBatch; ++u) {
-            const int64_t i = ib + (int64_t)u * kScatterThreads;
+            const int i = ib + u * kScatterThreads;
             const int e = ev[u];
-            // ids come from one complete selection; after an aborted one (a
-            // timed-out wait, reported in the status word) they may not:
-            // never index outside the arrays
+            // ids from an aborted selection may hold anything: stay in bounds
             if (i >= i1 || (unsigned)e >= (unsigned)E) continue;
-            const int64_t t = i / k;
-            const int j = (int)(t / 32 - w0), b = (int)(t & 31);
-            const int r = s_cb[e] + s_pre[e * C + j] + __popc(s_bits[e * C + j] & ((1u << b) - 1u));
-            if (pl) pl[i] = r;
-            if (rl && r >= 0 && r < Tk) rl[r] = (int)t;
+            const int t = lk >= 0 ? (i >> lk) : i / k;
+            const int sj = (e << lc) + (t >> 5) - (int)w0;
+            pl[i] = s_cb[e] + s_pre[sj] + __popc(s_bits[sj] & ((1u << (t & 31)) - 1u));
         }
     }
 }
@@ -206,6 +240,8 @@ cudaError_t launch_route_dispatch(const uint32_t *bits, const int *counts, const
                                   int *chunk_base, cudaStream_t s) {
     if (!offsets && !rows && !pos) return cudaSuccess;
     const int C = route_chunk_words(p);
+    int lc = 0;
+    while ((1 << lc) < C) ++lc;
     const int64_t nchunks = route_chunks(p);
     int *cb = (rows || pos) ? chunk_base : nullptr;
     cudaLaunchAttribute attr[1];
@@ -217,14 +253,15 @@ cudaError_t launch_route_dispatch(const uint32_t *bits, const int *counts, const
     cfg.stream = s;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, route_scan_kernel, bits, counts, p.E, p.W, C, nchunks,
-                                       offsets, cb);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, route_scan_kernel, bits, counts, p.E, p.W, lc,
+                                       nchunks, offsets, cb);
     if (e != cudaSuccess || !cb) return e;
     cfg.gridDim = dim3((unsigned)nchunks, (unsigned)p.L);
     cfg.blockDim = dim3(kScatterThreads);
     cfg.dynamicSmemBytes = sizeof(int) * (size_t)(2 * p.E * C + p.E);
-    return cudaLaunchKernelEx(&cfg, route_scatter_kernel, bits, ids, (const int *)cb, p.T, p.E,
-                              p.k, p.W, C, nchunks, rows, pos);
+    const int lk = (p.k & (p.k - 1)) == 0 ? __builtin_ctz((unsigned)p.k) : -1;
+    return cudaLaunchKernelEx(&cfg, route_scatter_kernel, bits, ids, (const int *)cb, (int)p.T,
+                              p.E, p.k, lk, p.W, lc, nchunks, rows, pos);
 }
 
 }  // namespace dol

@@ -43,6 +43,8 @@ EXPORTS = {
     "do_routing_workspace_size": (["i64", "i32", "i32", "i32"], "sz"),
     "do_forward_backward_routed": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p", "p",
                                     "p", "p", "p", "p", "p", "p", "p", "p", "p", "sz", "p"], "i32"),
+    "do_maxvio": (["p", "p", "i32", "i32", "i32", "p", "p", "p", "p"], "i32"),
+    "do_rem_allocate": (["p", "p", "p", "i32", "i32", "i32", "p", "p", "p", "p", "p", "p"], "i32"),
 }
 
 _CT = {"p": ctypes.c_void_p, "i64": ctypes.c_int64, "i32": ctypes.c_int32,
@@ -255,6 +257,51 @@ def forward_backward_routed(logits, k, gate=GATE_SIGMOID_NORM, grad_scale=1.0,
         _ptr(route.rows), _ptr(route.pos), out.workspace.data_ptr(), out.workspace.numel(),
         _stream(z)))
     return out, route
+
+
+def maxvio(counts: torch.Tensor, expert_rank: torch.Tensor, R: int, with_rank_loads=False,
+           status_flags: torch.Tensor | None = None):
+    """do_maxvio: MaxVio (App. E) of each problem's counts [L,E] (device int32)
+    for the expert-to-rank map expert_rank [E] (device int32).  Returns maxvio
+    [L] float64 (and rank_loads [L,R] int64 when asked)."""
+    if counts.dim() == 1:
+        counts = counts.unsqueeze(0)
+    L, E = counts.shape
+    if counts.dtype != torch.int32 or expert_rank.dtype != torch.int32:
+        raise ValueError("counts and expert_rank must be int32")
+    if not (counts.is_cuda and expert_rank.is_cuda and counts.is_contiguous()
+            and expert_rank.is_contiguous()) or expert_rank.numel() != E:
+        raise ValueError("counts [L,E] and expert_rank [E] must be contiguous CUDA tensors")
+    out = torch.empty(L, dtype=torch.float64, device=counts.device)
+    loads = torch.empty(L, R, dtype=torch.int64, device=counts.device) if with_rank_loads else None
+    _check("do_maxvio", lib().do_maxvio(counts.data_ptr(), expert_rank.data_ptr(), E, R, L,
+                                        _ptr(loads), out.data_ptr(), _ptr(status_flags),
+                                        _stream(counts)))
+    return (out, loads) if with_rank_loads else out
+
+
+def rem_allocate(loads, expert_tokens, expert_rank, D: int):
+    """do_rem_allocate (host): REM global-batch replica allocation.  Returns
+    (placements, loads_after): placements a list of (expert, sender, receiver,
+    tokens) in the order made, loads_after a float64 array [R]."""
+    import numpy as np
+
+    Lr = np.ascontiguousarray(loads, dtype=np.float64)
+    Te = np.ascontiguousarray(expert_tokens, dtype=np.float64)
+    er = np.ascontiguousarray(expert_rank, dtype=np.int32)
+    R, E = Lr.size, Te.size
+    if er.size != E:
+        raise ValueError("expert_rank must have one entry per expert")
+    cap = max(1, R * D)
+    pe, ps, pr = (np.zeros(cap, np.int32) for _ in range(3))
+    pt = np.zeros(cap, np.float64)
+    n = np.zeros(1, np.int32)
+    out = np.zeros(R, np.float64)
+    _check("do_rem_allocate", lib().do_rem_allocate(
+        Lr.ctypes.data, Te.ctypes.data, er.ctypes.data, R, E, D, pe.ctypes.data, ps.ctypes.data,
+        pr.ctypes.data, pt.ctypes.data, n.ctypes.data, out.ctypes.data))
+    k = int(n[0])
+    return [(int(pe[i]), int(ps[i]), int(pr[i]), float(pt[i])) for i in range(k)], out
 
 
 def device_status(workspace: torch.Tensor) -> int:
