@@ -66,6 +66,9 @@ def _load():
             "oracle_forward_backward": ([P, I64, I32, I32, I32, D, D, P, P, P, P, P, P], ctypes.c_int),
             "oracle_route": ([P, I64, I32, I32, I32, P, P], None),
             "oracle_dispatch": ([P, I64, I32, I32, P, P, P], None),
+            "oracle_bf16_to_double": ([P, I64, P], None),
+            "oracle_router_logits": ([P, P, I64, I32, I32, P], None),
+            "oracle_router_grad": ([P, P, P, I64, I32, I32, P, P], None),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -220,3 +223,36 @@ def dispatch(ids, E):
     pos = np.empty((T, k), np.int32)
     _load().oracle_dispatch(pi, T, E, k, offsets.ctypes.data, rows.ctypes.data, pos.ctypes.data)
     return offsets, rows, pos
+
+
+def bf16_to_double(h):
+    """Exact values of bf16 bit patterns (uint16 array)."""
+    h, ph = _c(h, np.uint16)
+    out = np.empty(h.shape, np.float64)
+    _load().oracle_bf16_to_double(ph, h.size, out.ctypes.data)
+    return out
+
+
+def router_logits(X, Wr):
+    """z [T,E] float64 = X Wr^T for bf16 bit patterns X [T,H], Wr [E,H] (uint16)."""
+    X, px = _c(X, np.uint16)
+    Wr, pw = _c(Wr, np.uint16)
+    T, H = X.shape
+    E = Wr.shape[0]
+    z = np.empty((T, E), np.float64)
+    _load().oracle_router_logits(px, pw, T, H, E, z.ctypes.data)
+    return z
+
+
+def router_grad(X, Wr, dz, with_dx=False):
+    """dW [E,H] (and dX [T,H]) float64 of z = X Wr^T for the upstream dz [T,E]."""
+    X, px = _c(X, np.uint16)
+    Wr, pw = _c(Wr, np.uint16)
+    dz, pd = _c(dz, np.float64)
+    T, H = X.shape
+    E = Wr.shape[0]
+    dW = np.empty((E, H), np.float64)
+    dX = np.empty((T, H), np.float64) if with_dx else None
+    _load().oracle_router_grad(px, pw, pd, T, H, E, dW.ctypes.data,
+                               dX.ctypes.data if dX is not None else None)
+    return (dW, dX) if with_dx else dW

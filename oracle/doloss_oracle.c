@@ -308,3 +308,54 @@ void oracle_dispatch(const int32_t *ids, int64_t T, int32_t E, int32_t k, int32_
         }
     free(fill);
 }
+
+/* bf16 is the upper half of an IEEE binary32: widening it is exact. */
+static double bf16_value(uint16_t h)
+{
+    uint32_t u = (uint32_t)h << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+void oracle_bf16_to_double(const uint16_t *h, int64_t n, double *out)
+{
+    for (int64_t i = 0; i < n; ++i) out[i] = bf16_value(h[i]);
+}
+
+/* The router that produces the logits of Eq. 1 (Sec. 4.1: a linear map from
+ * the hidden size to the n experts, no bias, as in the Qwen3-MoE architecture
+ * the paper trains): z_te = sum_h X_th W_eh, with X [T][H] and W [E][H] in
+ * bf16 and every product and sum in double.  z is [T][E]. */
+void oracle_router_logits(const uint16_t *X, const uint16_t *Wr, int64_t T, int32_t H, int32_t E,
+                          double *z)
+{
+    for (int64_t t = 0; t < T; ++t)
+        for (int32_t e = 0; e < E; ++e) {
+            double acc = 0.0;
+            for (int32_t h = 0; h < H; ++h)
+                acc += bf16_value(X[t * H + h]) * bf16_value(Wr[(int64_t)e * H + h]);
+            z[t * E + e] = acc;
+        }
+}
+
+/* Gradients of that linear map for an upstream gradient dz [T][E] (double):
+ * dW_eh = sum_t dz_te X_th ([E][H]) and, when dX is not NULL,
+ * dX_th = sum_e dz_te W_eh ([T][H]). */
+void oracle_router_grad(const uint16_t *X, const uint16_t *Wr, const double *dz, int64_t T,
+                        int32_t H, int32_t E, double *dW, double *dX)
+{
+    for (int32_t e = 0; e < E; ++e)
+        for (int32_t h = 0; h < H; ++h) {
+            double acc = 0.0;
+            for (int64_t t = 0; t < T; ++t) acc += dz[t * E + e] * bf16_value(X[t * H + h]);
+            dW[(int64_t)e * H + h] = acc;
+        }
+    if (!dX) return;
+    for (int64_t t = 0; t < T; ++t)
+        for (int32_t h = 0; h < H; ++h) {
+            double acc = 0.0;
+            for (int32_t e = 0; e < E; ++e) acc += dz[t * E + e] * bf16_value(Wr[(int64_t)e * H + h]);
+            dX[t * H + h] = acc;
+        }
+}
