@@ -160,6 +160,25 @@ do_status do_forward_backward_routed(const float *logits, int64_t T, int32_t E, 
                                      int32_t *dispatch_pos, void *workspace,
                                      size_t workspace_bytes, void *stream);
 
+/* Router-side fusion: the logits come from the router's linear map (Sec. 4.1:
+ * hidden size H to the E experts, no bias), computed here on the tensor cores
+ * from bf16 inputs with fp32 accumulation,
+ *   logits[l][t][e] = sum_h X[l][t][h] W[l][e][h],
+ * with step 1 (Top-K, signatures, co-occurrence counts) done on each tile of
+ * logits while it is still on chip; the logits are written to `logits`
+ * ([L][T][E] fp32, an output here) for the loss step, and everything else is
+ * as do_forward_backward.  X [L][T][H] and W [L][E][H] are bf16 (uint16 bit
+ * patterns), 16-byte aligned.  Supported: E = 128, k in {1, 2, 4, 8}, H a
+ * multiple of 64, logits 16-byte aligned and the conditions of the fused
+ * path of do_forward_backward (16-byte aligned bits and dlogits given);
+ * otherwise DO_ERR_UNSUPPORTED.  Same workspace as do_forward_backward.  The
+ * selection is taken on the fp32 logits this call writes. */
+do_status do_router_forward_backward(const void *X, const void *Wr, int64_t T, int32_t H, int32_t E,
+                                     int32_t k, int32_t L, int32_t gate, float grad_scale,
+                                     float *logits, uint32_t *bits, int32_t *counts, int32_t *D,
+                                     float *loss, int64_t *origin_do, float *dlogits,
+                                     void *workspace, size_t workspace_bytes, void *stream);
+
 /* Device workspace, in bytes, that do_loss_fwd_bwd and do_forward_backward
  * need for these sizes (0 if the sizes are invalid). */
 size_t do_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L);

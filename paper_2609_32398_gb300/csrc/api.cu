@@ -61,6 +61,14 @@ struct RouteArgs {
     int32_t *offsets, *rows, *pos;
 };
 
+// The router's inputs when the logits are computed in the fused path
+// (do_router_forward_backward): bf16 X [L][T][H] and W [L][E][H].
+struct RouterIn {
+    const void *X;
+    const void *Wr;
+    int H;
+};
+
 // Checks shared by the entry points that write routing outputs: the row and
 // token indices of the dispatch arrays are int32.
 do_status check_route(const Problem &p, const RouteArgs &r) {
@@ -185,7 +193,7 @@ do_status forward_backward_impl(const float *logits, int64_t T, int32_t E, int32
                                 int32_t *D, float *loss, int64_t *origin_do, float *dlogits,
                                 void *workspace, size_t workspace_bytes, void *stream,
                                 int *status_out, bool *status_done,
-                                const RouteArgs *ra = nullptr) {
+                                const RouteArgs *ra = nullptr, const RouterIn *rin = nullptr) {
     if (status_done) *status_done = false;
     Problem p;
     do_status st = check_sizes(T, E, k, L, &p);
@@ -202,8 +210,13 @@ do_status forward_backward_impl(const float *logits, int64_t T, int32_t E, int32
         return DO_ERR_WORKSPACE;
     cudaStream_t s = (cudaStream_t)stream;
     const dol::RouteOut route = {ra ? ra->ids : nullptr, ra ? ra->combine : nullptr, gate};
-    if (dol::signatures_fast_supported(logits, p) && dol::loss_fast_supported(p, logits, D, dlogits) &&
-        aligned(bits, 16) && route_fast_ok(ra)) {
+    const bool fast = dol::signatures_fast_supported(logits, p) &&
+                      dol::loss_fast_supported(p, logits, D, dlogits) && aligned(bits, 16) &&
+                      route_fast_ok(ra);
+    // the router GEMM runs only in the fused fast path, without routing outputs
+    if (rin && !(fast && !ra && dol::router_supported(p, rin->H, rin->X, rin->Wr, logits)))
+        return DO_ERR_UNSUPPORTED;
+    if (fast) {
         // signatures (+ per-CTA co-occurrence counts) -> reduction to C -> loss,
         // which builds D = n_i + n_j - 2 c_ij and writes D and the counts
         const dol::WsLayout w = dol::ws_layout(p);
@@ -224,12 +237,15 @@ do_status forward_backward_impl(const float *logits, int64_t T, int32_t E, int32
                          dol::loss_mma_supported(p, gate, logits, D, dlogits);
         unsigned char *bimg = mma ? reinterpret_cast<unsigned char *>(ws + w.bimg) : nullptr;
         cudaError_t e =
-            ra ? dol::launch_signatures_fast_routed(logits, p, bits, n_acc, idx, parts, zero, status,
-                                                    route, s)
-               : dol::launch_signatures_fast(logits, p, bits, n_acc, idx, parts, zero, status, s);
+            rin ? dol::launch_router_signatures(rin->X, rin->Wr, rin->H, const_cast<float *>(logits),
+                                                p, bits, n_acc, idx, parts, zero, status, s)
+            : ra ? dol::launch_signatures_fast_routed(logits, p, bits, n_acc, idx, parts, zero,
+                                                      status, route, s)
+                 : dol::launch_signatures_fast(logits, p, bits, n_acc, idx, parts, zero, status, s);
+        const int P1 = rin ? dol::router_ctas_per_problem(p) : dol::sig_fast_ctas_per_problem(p);
         if (e == cudaSuccess)
-            e = dol::launch_cooc_reduce(parts, dol::sig_fast_ctas_per_problem(p), n_acc, p, D,
-                                        counts, bimg, reinterpret_cast<long long *>(origin_do), s);
+            e = dol::launch_cooc_reduce(parts, P1, n_acc, p, D, counts, bimg,
+                                        reinterpret_cast<long long *>(origin_do), s);
         if (e == cudaSuccess) {
             if (mma)
                 e = dol::launch_loss_mma(logits, idx, bimg, n_acc, p, 1.0f, grad_scale, loss, dlogits,
@@ -286,6 +302,20 @@ do_status do_forward_backward_routed(const float *logits, int64_t T, int32_t E, 
     return forward_backward_impl(logits, T, E, k, L, gate, grad_scale, bits, counts, D, loss,
                                  origin_do, dlogits, workspace, workspace_bytes, stream, nullptr,
                                  nullptr, &ra);
+}
+
+do_status do_router_forward_backward(const void *X, const void *Wr, int64_t T, int32_t H, int32_t E,
+                                     int32_t k, int32_t L, int32_t gate, float grad_scale,
+                                     float *logits, uint32_t *bits, int32_t *counts, int32_t *D,
+                                     float *loss, int64_t *origin_do, float *dlogits,
+                                     void *workspace, size_t workspace_bytes, void *stream) {
+    NvtxRange nvtx("do_router_forward_backward");
+    if (!X || !Wr || !logits) return DO_ERR_INVALID_ARG;
+    if (H < 1) return DO_ERR_INVALID_ARG;
+    const RouterIn rin = {X, Wr, H};
+    return forward_backward_impl(logits, T, E, k, L, gate, grad_scale, bits, counts, D, loss,
+                                 origin_do, dlogits, workspace, workspace_bytes, stream, nullptr,
+                                 nullptr, nullptr, &rin);
 }
 
 do_status do_routing(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L, int32_t gate,

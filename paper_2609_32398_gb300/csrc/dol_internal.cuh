@@ -98,6 +98,16 @@ int64_t route_chunks(const Problem &p);
 cudaError_t launch_route_dispatch(const uint32_t *bits, const int *counts, const int *ids,
                                   const Problem &p, int *offsets, int *rows, int *pos,
                                   int *chunk_base, cudaStream_t s);
+// Router-side fusion (E = 128, k in {1,2,4,8}, H a multiple of 64, 16-byte
+// aligned X, W and logits): logits = X W^T on the tensor cores with the
+// fused path's signature step in the epilogue (bits, selected indices,
+// per-CTA co-occurrence triangles, counts accumulated into `counts`).
+bool router_supported(const Problem &p, int H, const void *X, const void *Wr, const float *logits);
+int router_ctas_per_problem(const Problem &p);
+cudaError_t launch_router_signatures(const void *X, const void *Wr, int H, float *logits,
+                                     const Problem &p, uint32_t *bits, int *counts, uint8_t *idx,
+                                     uint32_t *cooc, const ZeroSpans &zero, int *status,
+                                     cudaStream_t s);
 bool loss_fast_supported(const Problem &p, const float *logits, const int *D, const float *dlogits);
 cudaError_t launch_idx_from_bits(const uint32_t *bits, const Problem &p, uint8_t *idx, int *zero_ptr,
                                  int zero_n, cudaStream_t s);

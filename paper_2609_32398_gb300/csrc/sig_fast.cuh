@@ -119,6 +119,124 @@ __device__ __forceinline__ void store_route(const RouteOut &r, int64_t off, cons
     }
 }
 
+// Top-K of the token held by this lane in a swizzled 32-token tile (the layout
+// of chunk_ptr): the row is cut into NG groups of GS experts whose maxima are
+// kept in registers; K times a tournament over the group maxima (ties to the
+// lower group) picks a group, the first element equal to its maximum is chosen
+// (lowest index among equal values), overwritten with -inf in the tile, and
+// the group maximum recomputed.  sel: the chosen experts in selection order;
+// val: their logits.
+template <int E, int K>
+__device__ __forceinline__ void select_topk(unsigned char *tp, int lane, int (&sel)[K],
+                                            float (&val)[K]) {
+    constexpr int GS = SigCfg<E>::GS, NG = SigCfg<E>::NG, GS4 = GS / 4;
+    float g[NG];
+#pragma unroll
+    for (int gi = 0; gi < NG; ++gi) {
+        float m = -INFINITY;
+#pragma unroll
+        for (int c = 0; c < GS4; ++c) {
+            const float4 v = *reinterpret_cast<const float4 *>(chunk_ptr(tp, gi * GS4 + c, lane));
+            m = fmaxf(m, fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w)));
+        }
+        g[gi] = m;
+    }
+#pragma unroll
+    for (int qk = 0; qk < K; ++qk) {
+        float tv[NG];
+        int ti[NG];
+#pragma unroll
+        for (int j = 0; j < NG / 2; ++j) {
+            const bool right = g[2 * j + 1] > g[2 * j];
+            tv[j] = right ? g[2 * j + 1] : g[2 * j];
+            ti[j] = right ? 2 * j + 1 : 2 * j;
+        }
+#pragma unroll
+        for (int nn = NG / 2; nn > 1; nn >>= 1) {
+#pragma unroll
+            for (int j = 0; j < nn / 2; ++j) {
+                const bool right = tv[2 * j + 1] > tv[2 * j];
+                tv[j] = right ? tv[2 * j + 1] : tv[2 * j];
+                ti[j] = right ? ti[2 * j + 1] : ti[2 * j];
+            }
+        }
+        const float bv = tv[0];
+        const int bi = ti[0];
+        float x[GS];
+#pragma unroll
+        for (int c = 0; c < GS4; ++c) {
+            const float4 v = *reinterpret_cast<const float4 *>(chunk_ptr(tp, bi * GS4 + c, lane));
+            x[4 * c] = v.x;
+            x[4 * c + 1] = v.y;
+            x[4 * c + 2] = v.z;
+            x[4 * c + 3] = v.w;
+        }
+        int p = GS - 1;
+#pragma unroll
+        for (int j = GS - 1; j >= 0; --j)
+            if (x[j] == bv) p = j;
+        float m2 = -INFINITY;
+#pragma unroll
+        for (int j = 0; j < GS; ++j) m2 = fmaxf(m2, j == p ? -INFINITY : x[j]);
+        const int e = bi * GS + p;
+        reinterpret_cast<float *>(chunk_ptr(tp, e >> 2, lane))[e & 3] = -INFINITY;
+#pragma unroll
+        for (int gi = 0; gi < NG; ++gi) g[gi] = (gi == bi) ? m2 : g[gi];
+        sel[qk] = e;
+        val[qk] = bv;
+    }
+}
+
+// c_ab += 1 for every pair a < b of one token's chosen experts, in a
+// shared-memory triangle whose row a starts at s_rowoff[a] (the counts on the
+// diagonal come from the signature words).
+template <int K>
+__device__ __forceinline__ void cooc_add(uint32_t *s_cooc, const int *s_rowoff, const int (&sel)[K]) {
+    int so[K];
+#pragma unroll
+    for (int q = 0; q < K; ++q) so[q] = sel[q];
+#pragma unroll
+    for (int i = 1; i < K; ++i)  // insertion sort of K indices (static network)
+#pragma unroll
+        for (int j = i; j > 0; --j) {
+            const int lo = min(so[j - 1], so[j]), hi = max(so[j - 1], so[j]);
+            so[j - 1] = lo;
+            so[j] = hi;
+        }
+#pragma unroll
+    for (int q1 = 0; q1 < K - 1; ++q1) {
+        uint32_t *row = s_cooc + s_rowoff[so[q1]];
+#pragma unroll
+        for (int q2 = q1 + 1; q2 < K; ++q2) atomicAdd(row + so[q2], 1u);
+    }
+}
+
+// The signature words of the warp's 32 tokens (lane = token): a bit per chosen
+// expert, turned into one word per expert by 32x32 bit transposes; lane c
+// stores the word of expert 32 r + c at words[(32 r + c) W].  With kCount,
+// cnt[r] accumulates the word's population count.
+template <int E, int K, bool kCount>
+__device__ __forceinline__ void emit_words(const int (&sel)[K], bool valid, int lane,
+                                           uint32_t *words, int64_t W, uint32_t (&cnt)[E / 32]) {
+    constexpr int R = E / 32;
+    uint32_t m[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) m[r] = 0u;
+#pragma unroll
+    for (int qk = 0; qk < K; ++qk) {
+        const uint32_t bit = 1u << (sel[qk] & 31);
+        const int rq = sel[qk] >> 5;
+#pragma unroll
+        for (int r = 0; r < R; ++r) m[r] |= (rq == r) ? bit : 0u;
+    }
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+        const uint32_t word = transpose32(valid ? m[r] : 0u, lane);
+        words[(int64_t)(32 * r + lane) * W] = word;
+        if (kCount) cnt[r] += __popc(word);
+    }
+}
+
 template <int E, int K, bool kCounts, bool kCooc, bool kRoute>
 __global__ void __launch_bounds__(kFastThreads, 1)
 sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W,
@@ -205,7 +323,6 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W,
 
     // consumers
     constexpr int R = E / 32;
-    constexpr int GS = C::GS, NG = C::NG, GS4 = GS / 4;
     uint32_t cnt[R];
 #pragma unroll
     for (int r = 0; r < R; ++r) cnt[r] = 0u;
@@ -235,65 +352,9 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W,
         const bool valid = t < T;
         unsigned char *tp = smem + (size_t)s * C::kTileBytes;
 
-        // 1. group maxima
-        float g[NG];
-#pragma unroll
-        for (int gi = 0; gi < NG; ++gi) {
-            float m = -INFINITY;
-#pragma unroll
-            for (int c = 0; c < GS4; ++c) {
-                const float4 v = *reinterpret_cast<const float4 *>(chunk_ptr(tp, gi * GS4 + c, lane));
-                m = fmaxf(m, fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w)));
-            }
-            g[gi] = m;
-        }
-        // 2. K extractions
         int sel[K];
         float val[K];  // the chosen logits (kRoute)
-#pragma unroll
-        for (int qk = 0; qk < K; ++qk) {
-            float tv[NG];
-            int ti[NG];
-#pragma unroll
-            for (int j = 0; j < NG / 2; ++j) {
-                const bool right = g[2 * j + 1] > g[2 * j];
-                tv[j] = right ? g[2 * j + 1] : g[2 * j];
-                ti[j] = right ? 2 * j + 1 : 2 * j;
-            }
-#pragma unroll
-            for (int nn = NG / 2; nn > 1; nn >>= 1) {
-#pragma unroll
-                for (int j = 0; j < nn / 2; ++j) {
-                    const bool right = tv[2 * j + 1] > tv[2 * j];
-                    tv[j] = right ? tv[2 * j + 1] : tv[2 * j];
-                    ti[j] = right ? ti[2 * j + 1] : ti[2 * j];
-                }
-            }
-            const float bv = tv[0];
-            const int bi = ti[0];
-            float x[GS];
-#pragma unroll
-            for (int c = 0; c < GS4; ++c) {
-                const float4 v = *reinterpret_cast<const float4 *>(chunk_ptr(tp, bi * GS4 + c, lane));
-                x[4 * c] = v.x;
-                x[4 * c + 1] = v.y;
-                x[4 * c + 2] = v.z;
-                x[4 * c + 3] = v.w;
-            }
-            int p = GS - 1;
-#pragma unroll
-            for (int j = GS - 1; j >= 0; --j)
-                if (x[j] == bv) p = j;
-            float m2 = -INFINITY;
-#pragma unroll
-            for (int j = 0; j < GS; ++j) m2 = fmaxf(m2, j == p ? -INFINITY : x[j]);
-            const int e = bi * GS + p;
-            reinterpret_cast<float *>(chunk_ptr(tp, e >> 2, lane))[e & 3] = -INFINITY;
-#pragma unroll
-            for (int gi = 0; gi < NG; ++gi) g[gi] = (gi == bi) ? m2 : g[gi];
-            sel[qk] = e;
-            val[qk] = bv;
-        }
+        select_topk<E, K>(tp, lane, sel, val);
         // the tile is no longer read: hand the slot back to the producer
         fence_proxy_async_smem();
         __syncwarp();
@@ -301,43 +362,8 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W,
 
         if (idx && valid) store_idx<K>(idx + (layer * T + t) * K, sel);
         if (kRoute && valid) store_route<K>(route, (layer * T + t) * K, sel, val);
-        if (kCooc && valid) {
-            // c_ab += 1 for every pair a < b of selected experts (the counts on
-            // the diagonal come from the signature words below)
-            int so[K];
-#pragma unroll
-            for (int q = 0; q < K; ++q) so[q] = sel[q];
-#pragma unroll
-            for (int i = 1; i < K; ++i)  // insertion sort of K indices (static network)
-#pragma unroll
-                for (int j = i; j > 0; --j) {
-                    const int lo = min(so[j - 1], so[j]), hi = max(so[j - 1], so[j]);
-                    so[j - 1] = lo;
-                    so[j] = hi;
-                }
-#pragma unroll
-            for (int q1 = 0; q1 < K - 1; ++q1) {
-                uint32_t *row = s_cooc + s_rowoff[so[q1]];
-#pragma unroll
-                for (int q2 = q1 + 1; q2 < K; ++q2) atomicAdd(row + so[q2], 1u);
-            }
-        }
-        uint32_t m[R];
-#pragma unroll
-        for (int r = 0; r < R; ++r) m[r] = 0u;
-#pragma unroll
-        for (int qk = 0; qk < K; ++qk) {
-            const uint32_t bit = 1u << (sel[qk] & 31);
-            const int rq = sel[qk] >> 5;
-#pragma unroll
-            for (int r = 0; r < R; ++r) m[r] |= (rq == r) ? bit : 0u;
-        }
-#pragma unroll
-        for (int r = 0; r < R; ++r) {
-            const uint32_t word = transpose32(valid ? m[r] : 0u, lane);
-            bits[(layer * E + 32 * r + lane) * W + w] = word;
-            if (kCounts || kCooc) cnt[r] += __popc(word);
-        }
+        if (kCooc && valid) cooc_add<K>(s_cooc, s_rowoff, sel);
+        emit_words<E, K, kCounts || kCooc>(sel, valid, lane, bits + layer * E * W + w, W, cnt);
     }
     if (kCounts) {
 #pragma unroll

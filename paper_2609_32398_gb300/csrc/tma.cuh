@@ -257,4 +257,10 @@ __device__ __forceinline__ uint64_t umma_desc_sw128(uint32_t addr) {
 bool encode_tensor_map_3d_f32(CUtensorMap *map, const float *base, uint64_t planes, uint64_t rows,
                               uint64_t cols, uint32_t box_rows);
 
+// Host: 3-D bf16 tensor map over [planes][rows][cols] (cols innermost), box
+// box_cols x box_rows x 1 (box_cols * 2 bytes <= 128), 128-byte swizzle;
+// positions outside the tensor read as zero.
+bool encode_tensor_map_3d_bf16(CUtensorMap *map, const void *base, uint64_t planes, uint64_t rows,
+                               uint64_t cols, uint32_t box_cols, uint32_t box_rows);
+
 }  // namespace dol

@@ -44,6 +44,8 @@ EXPORTS = {
     "do_forward_backward_routed": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p", "p",
                                     "p", "p", "p", "p", "p", "p", "p", "p", "p", "sz", "p"], "i32"),
     "do_maxvio": (["p", "p", "i32", "i32", "i32", "p", "p", "p", "p"], "i32"),
+    "do_router_forward_backward": (["p", "p", "i64", "i32", "i32", "i32", "i32", "i32", "f32", "p",
+                                    "p", "p", "p", "p", "p", "p", "p", "sz", "p"], "i32"),
     "do_rem_allocate": (["p", "p", "p", "i32", "i32", "i32", "p", "p", "p", "p", "p", "p"], "i32"),
 }
 
@@ -257,6 +259,38 @@ def forward_backward_routed(logits, k, gate=GATE_SIGMOID_NORM, grad_scale=1.0,
         _ptr(route.rows), _ptr(route.pos), out.workspace.data_ptr(), out.workspace.numel(),
         _stream(z)))
     return out, route
+
+
+def router_forward_backward(X: torch.Tensor, Wr: torch.Tensor, k, gate=GATE_SIGMOID_NORM,
+                            grad_scale=1.0, out: Buffers | None = None,
+                            logits: torch.Tensor | None = None):
+    """do_router_forward_backward: logits = X Wr^T (bf16 X [L,T,H] or [T,H],
+    Wr [L,E,H] or [E,H]) on the tensor cores, then steps 1-3.  Returns
+    (logits [L,T,E] fp32, Buffers)."""
+    if X.dim() == 2:
+        X = X.unsqueeze(0)
+    if Wr.dim() == 2:
+        Wr = Wr.unsqueeze(0)
+    if X.dtype != torch.bfloat16 or Wr.dtype != torch.bfloat16 or not (X.is_cuda and Wr.is_cuda):
+        raise ValueError("X and Wr must be CUDA bfloat16 tensors")
+    if not (X.is_contiguous() and Wr.is_contiguous()):
+        raise ValueError("X and Wr must be contiguous")
+    L, T, H = X.shape
+    if Wr.shape[0] != L or Wr.shape[2] != H:
+        raise ValueError("Wr must be [L, E, H] for X [L, T, H]")
+    E = Wr.shape[1]
+    if logits is None:
+        logits = torch.empty(L, T, E, dtype=torch.float32, device=X.device)
+    if out is None:
+        out = Buffers(L, T, E, k, X.device)
+    if out.shape != (L, T, E, k):
+        raise ValueError("output buffers were made for another shape")
+    _check("do_router_forward_backward", lib().do_router_forward_backward(
+        X.data_ptr(), Wr.data_ptr(), T, H, E, k, L, gate, grad_scale, logits.data_ptr(),
+        out.bits.data_ptr(), out.counts.data_ptr(), out.D.data_ptr(), out.loss.data_ptr(),
+        out.origin_do.data_ptr(), _ptr(out.dlogits), out.workspace.data_ptr(),
+        out.workspace.numel(), _stream(X)))
+    return logits, out
 
 
 def maxvio(counts: torch.Tensor, expert_rank: torch.Tensor, R: int, with_rank_loads=False,

@@ -125,3 +125,12 @@ def random_logits(T: int, E: int, L: int = 1, seed: int = 0, device="cpu",
     if ties:
         z = torch.round(z * 2.0) / 2.0
     return z
+
+
+def router_inputs(T: int, H: int, E: int = 128, L: int = 1, seed: int = 0, device="cpu"):
+    """Router inputs in the c3 recipe's distribution: hidden states X [L,T,H]
+    ~N(0,1) and router weights W [L,E,H] ~N(0,0.02), both rounded to bf16."""
+    g = _gen(device, seed)
+    X = torch.randn(L, T, H, generator=g, device=device).to(torch.bfloat16)
+    W = (torch.randn(L, E, H, generator=g, device=device) * 0.02).to(torch.bfloat16)
+    return X, W

@@ -108,3 +108,17 @@ def test_routing_entry_points_validate_on_the_host(dl):
     assert lib.do_forward_backward_routed(fake, 64, 8, 2, 1, 0, 1.0, fake, fake, fake, fake, None,
                                           None, fake, fake, None, None, None, fake, 8,
                                           None) == WS
+
+
+def test_router_entry_point_validates_on_the_host(dl):
+    lib = dl.lib()
+    fake = ctypes.c_void_p(0x10000)
+    INV, UNS = 1, 2
+    big = 1 << 30
+    args = lambda X, T, H, E, k: (X, fake, T, H, E, k, 1, 0, 1.0, fake, fake, fake, fake, fake,
+                                  None, fake, fake, big, None)
+    assert lib.do_router_forward_backward(*args(None, 1024, 256, 128, 8)) == INV
+    assert lib.do_router_forward_backward(*args(fake, 1024, 0, 128, 8)) == INV    # H = 0
+    assert lib.do_router_forward_backward(*args(fake, 1024, 256, 64, 8)) == UNS   # E != 128
+    assert lib.do_router_forward_backward(*args(fake, 1024, 96, 128, 8)) == UNS   # H % 64
+    assert lib.do_router_forward_backward(*args(fake, 1024, 256, 128, 3)) == UNS  # k
