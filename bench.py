@@ -63,6 +63,17 @@ def routing_bytes(T, E, k, L=1):
     return L * (4 * T * E + 16 * T * k + 8 * E + 4)
 
 
+ROUTER_HIDDEN = 2048  # the 30BA3B router's input width (hidden size, Sec. 4.1)
+
+
+def router_bytes(T, E, H, L=1):
+    """Bytes of the router-fused step: X and W read (2TH + 2EH bf16), the
+    logits written and read back once (8TE), dlogits written (4TE), and the
+    signature, Hamming-matrix and count traffic of the DO-loss path."""
+    W = (T + 31) // 32
+    return L * (2 * T * H + 2 * E * H + 12 * T * E + 8 * E * W + 8 * E * E + 4 * E)
+
+
 def measured_peaks():
     try:
         return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
@@ -275,6 +286,13 @@ def run_ours(args, rank, world, local):
         # (used under ncu)
         if args.quick_path == "loss":
             call, ws = step, sets[0][1].workspace
+        elif args.quick_path == "router":
+            X, Wr = workloads.router_inputs(T, ROUTER_HIDDEN, E, L, seed=w.seed, device=dev)
+            zr = torch.empty(L, T, E, dtype=torch.float32, device=dev)
+
+            def call(i):
+                dl.router_forward_backward(X, Wr, k, w.gate, 1.0, out=sets[0][1], logits=zr)
+            ws = sets[0][1].workspace
         else:
             route = dl.Routing(L, T, E, k, dev)
             if args.quick_path == "routing":
@@ -377,6 +395,37 @@ def run_ours(args, rank, world, local):
             st = dl.device_status(ws)
             if st != 0:
                 raise RuntimeError(f"device status after the routing runs: {dl.status_string(st)}")
+    # Router-side fusion: the router's linear map on the tensor cores with the
+    # signature step in its epilogue, then the rest of the path.  X (256 MiB of
+    # bf16 at H = 2048) is larger than L2 by itself.  Beside it, for context:
+    # cuBLAS's bf16 product (bf16 out) followed by the fused path on logits.
+    X, Wr = workloads.router_inputs(T, ROUTER_HIDDEN, E, L, seed=w.seed, device=dev)
+    zr = torch.empty(L, T, E, dtype=torch.float32, device=dev)
+    rout = sets[0][1]
+    for _ in range(3):
+        dl.router_forward_backward(X, Wr, k, w.gate, 1.0, out=rout, logits=zr)
+    torch.cuda.synchronize()
+    router_reps = max(20, min(args.steps, 500))
+    ra_, rb_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ra_.record(stream)
+    for _ in range(router_reps):
+        dl.router_forward_backward(X, Wr, k, w.gate, 1.0, out=rout, logits=zr)
+    rb_.record(stream)
+    torch.cuda.synchronize()
+    router_ms = ra_.elapsed_time(rb_) / router_reps
+    st = dl.device_status(rout.workspace)
+    if st != 0:
+        raise RuntimeError(f"device status after the router runs: {dl.status_string(st)}")
+    for _ in range(3):
+        torch.matmul(X[0], Wr[0].T)
+    ra_.record(stream)
+    for _ in range(router_reps):
+        torch.matmul(X[0], Wr[0].T)
+    rb_.record(stream)
+    torch.cuda.synchronize()
+    cublas_ms = ra_.elapsed_time(rb_) / router_reps
+    del X, Wr, zr
+
     peaks = measured_peaks()
     peak = peaks["hbm_gbs"] if peaks else 6800.0
     peak_src = "of measured" if peaks else "of fallback"
@@ -452,6 +501,21 @@ def run_ours(args, rank, world, local):
                           "us_per_call": routed_ms * 1e3,
                           "us_per_call_without_routing": plain_ms * 1e3},
                 "reps": reps},
+            "router_fused": {
+                "entry": "do_router_forward_backward (logits = X W^T on tcgen05 with the signature "
+                         "step in the GEMM epilogue, then the D reduction and the loss)",
+                "hidden": ROUTER_HIDDEN, "x_dtype": "bf16",
+                "us_per_call": router_ms * 1e3, "tokens_per_s": T * L / (router_ms * 1e-3),
+                "roofline": {"bound": "hbm", "kernel": "do_router_forward_backward",
+                             "achieved": router_bytes(T, E, ROUTER_HIDDEN, L) / (router_ms * 1e-3) / 1e9,
+                             "peak": peak, "unit": "GB/s",
+                             "frac": router_bytes(T, E, ROUTER_HIDDEN, L) / (router_ms * 1e-3) / 1e9 / peak,
+                             "peak_source": peak_src,
+                             "algorithmic_bytes": router_bytes(T, E, ROUTER_HIDDEN, L),
+                             "traffic": profiled_traffic("do_router_forward_backward")},
+                "context_unfused_us": {"cublas_bf16_matmul": cublas_ms * 1e3,
+                                       "do_forward_backward": plain_ms * 1e3},
+                "reps": router_reps},
             "clocks": clocks, "e2e": e2e, "gpu_launches": KERNELS_PER_STEP * args.steps,
             "cpu_baseline": cpu,
         }
@@ -467,9 +531,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--quick", action="store_true",
                     help="run warmup+steps plain steps and exit (for profilers)")
-    ap.add_argument("--quick-path", choices=["loss", "routing", "routed"], default="loss",
-                    help="entry point of --quick: do_forward_backward, do_routing or "
-                         "do_forward_backward_routed")
+    ap.add_argument("--quick-path", choices=["loss", "routing", "routed", "router"], default="loss",
+                    help="entry point of --quick: do_forward_backward, do_routing, "
+                         "do_forward_backward_routed or do_router_forward_backward")
     args = ap.parse_args()
     if args.impl == "reference":
         rank = int(os.environ.get("RANK", "0"))

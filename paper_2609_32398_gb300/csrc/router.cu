@@ -6,37 +6,45 @@
 // The logits are written once, for the loss kernel, and never read back for
 // the selection.
 //
-// One persistent CTA per SM walks 128-token tiles:
+// One persistent CTA per SM owns a contiguous, balanced range of 32-token
+// signature words (13 or 14 words for T = 65536 on 152 SMs) and walks it in
+// pair tiles of up to eight words (two 128-token MMA tiles that share one
+// slice of W):
 //   warp 0   TMA producer: per 64-wide slice of the hidden size, one X box
-//            [128 tokens x 64] and one W box [128 experts x 64] (bf16, 128-byte
-//            swizzle) into a 4-stage ring;
-//   warp 1   MMA issuer: 4 x tcgen05.mma kind::f16 (bf16 A and B, K = 16) per
-//            stage into one of two TMEM accumulators [128 lanes x 128 fp32];
-//   warps 2-5 epilogue, one TMEM lane quarter (32 tokens) each: the tile's
-//            logits go TMEM -> registers -> a swizzled shared-memory tile (the
-//            signature kernel's layout), out to HBM by TMA stores, and the
-//            signature kernel's per-token selection, co-occurrence counts and
-//            signature words run on that tile.
+//            [32 tokens x 64] per word and one W box [128 experts x 64] (bf16,
+//            128-byte swizzle) into a 3-stage ring (48 KB a stage, 32 KB of it
+//            X, so each SM keeps 96 KB of X in flight);
+//   warp 1   MMA issuer: per stage 2 x 4 tcgen05.mma kind::f16 (bf16, K = 16)
+//            into the two accumulators [128 lanes x 128 fp32] of the pair,
+//            double-buffered (all 512 TMEM columns);
+//   warps 2-5 epilogue, one TMEM lane quarter each (the same 32 rows of both
+//            tiles): the logits go TMEM -> registers -> a swizzled shared-memory
+//            tile (the signature kernel's layout), out to HBM by TMA stores, and
+//            the signature kernel's per-token selection and signature words run
+//            on that tile.  The co-occurrence counts go straight to this CTA's
+//            partial triangle in global memory (L2 reductions): shared memory
+//            is kept for the ring.
 #include "sig_fast.cuh"
 
 namespace dol {
 namespace {
 
 constexpr int kRE = 128;                        // experts = N of the MMA
-constexpr int kRTileM = 128;                    // tokens per tile = M of the MMA
+constexpr int kRTileM = 128;                    // tokens per MMA tile = M
+constexpr int kRPairWords = 8;                  // signature words of a pair tile (2 x 128 tokens)
 constexpr int kRSlice = 64;                     // hidden columns per stage (128 bytes of bf16)
-constexpr int kRStages = 4;
-constexpr int kRBoxBytes = kRTileM * 128;       // one 128-row box of 128 bytes
-constexpr int kRStageBytes = 2 * kRBoxBytes;    // X box + W box
+constexpr int kRStages = 3;
+constexpr int kRWordBox = 32 * 128;             // the X box of one signature word (32 rows)
+constexpr int kRTileBytes = kRTileM * 128;      // one MMA tile's A slice, or the W slice
+constexpr int kRStageBytes = 3 * kRTileBytes;   // X of two tiles + W
 constexpr int kREpiWarps = 4;
 constexpr int kRThreads = (2 + kREpiWarps) * 32;
 constexpr int kRZTileBytes = 32 * kRE * 4;      // one warp's 32 tokens x 128 logits
-constexpr int kRTmemCols = 2 * kRE;             // two fp32 accumulators
+constexpr int kRTmemCols = 4 * kRE;             // two buffers x two fp32 accumulators
 using RC = SigCfg<kRE>;
 
 constexpr size_t kROffZ = (size_t)kRStages * kRStageBytes;
-constexpr size_t kROffCooc = kROffZ + (size_t)kREpiWarps * kRZTileBytes;
-constexpr size_t kROffRowoff = kROffCooc + (size_t)RC::kCoocWords * 4;
+constexpr size_t kROffRowoff = kROffZ + (size_t)kREpiWarps * kRZTileBytes;
 constexpr size_t kROffBars = kROffRowoff + (size_t)kRE * 4;
 constexpr size_t kRNumBars = 2 * kRStages + 4;
 constexpr size_t kROffScal = kROffBars + kRNumBars * 8;
@@ -45,7 +53,6 @@ constexpr size_t kRSmem = kROffScal + 16 + 1024;  // + alignment slack of the ba
 struct RouterArgs {
     int64_t T, W;
     int H;
-    int ntiles;
     uint32_t *bits;
     uint8_t *idx;
     uint32_t *cooc;
@@ -53,6 +60,12 @@ struct RouterArgs {
     ZeroSpans zero;
     int *status;
 };
+
+// Words of the next tile of a range with r words left: pairs of MMA tiles
+// (eight words) that share each slice of W, the remainder last.
+__device__ __forceinline__ int next_tile_words(int64_t r) {
+    return r < kRPairWords ? (int)r : kRPairWords;
+}
 
 template <int K>
 __global__ void __launch_bounds__(kRThreads, 1)
@@ -63,7 +76,6 @@ router_sig_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constan
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     unsigned char *ring = smem;
     unsigned char *ztiles = smem + kROffZ;
-    uint32_t *s_cooc = reinterpret_cast<uint32_t *>(smem + kROffCooc);
     int *s_rowoff = reinterpret_cast<int *>(smem + kROffRowoff);
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kROffBars);
     uint64_t *full = bars, *empty = bars + kRStages;
@@ -75,9 +87,13 @@ router_sig_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constan
     const int layer = blockIdx.y;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nkb = a.H / kRSlice;
+    // this CTA's signature words [wb, we): an even split of the problem's W words
+    const int64_t wb = (int64_t)blockIdx.x * a.W / gridDim.x;
+    const int64_t we = (int64_t)(blockIdx.x + 1) * a.W / gridDim.x;
+    // this CTA's co-occurrence triangle (the reduction kernel's input)
+    uint32_t *tri = a.cooc + ((size_t)layer * gridDim.x + blockIdx.x) * (size_t)RC::kCoocWords;
     // Shared-memory and TMEM set-up touch no global memory: they overlap the
     // end of the previous kernel on the stream.
-    for (int i = threadIdx.x; i < RC::kCoocWords; i += kRThreads) s_cooc[i] = 0u;
     for (int e = threadIdx.x; e < kRE; e += kRThreads) s_rowoff[e] = cooc_row_offset<kRE>(e) - (e & ~3);
     if (threadIdx.x == 0) {
         for (int s = 0; s < kRStages; ++s) {
@@ -109,20 +125,30 @@ router_sig_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constan
         for (int64_t i = (int64_t)blockIdx.x * kRThreads + threadIdx.x; i < a.zero.n[z];
              i += (int64_t)gridDim.x * kRThreads)
             a.zero.p[z][i] = 0;
+    {  // the triangle starts at zero; the barrier below orders these stores
+       // before the reductions of the epilogue
+        uint4 *t4 = reinterpret_cast<uint4 *>(tri);
+        for (int q = threadIdx.x; q < RC::kCoocWords / 4; q += kRThreads) t4[q] = make_uint4(0u, 0u, 0u, 0u);
+    }
+    __syncthreads();
 
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
             int g = 0;
-            for (int m = blockIdx.x; m < a.ntiles && !*s_abort; m += gridDim.x) {
+            for (int64_t wt = wb, nw = 0; wt < we && !*s_abort; wt += nw) {
+                nw = next_tile_words(we - wt);
                 for (int kb = 0; kb < nkb; ++kb, ++g) {
                     const int s = g % kRStages, r = g / kRStages;
                     if (r > 0 && !mbar_wait(&empty[s], (uint32_t)(r - 1) & 1u, a.status)) *s_abort = 1;
                     if (*s_abort) break;
                     unsigned char *st = ring + (size_t)s * kRStageBytes;
-                    mbar_arrive_expect_tx(&full[s], kRStageBytes);
-                    tma_load_3d(st, &xmap, kb * kRSlice, m * kRTileM, layer, &full[s]);
-                    tma_load_3d(st + kRBoxBytes, &wmap, kb * kRSlice, 0, layer, &full[s]);
+                    // rows of missing words keep stale data: their outputs are not used
+                    mbar_arrive_expect_tx(&full[s], (uint32_t)((int)nw * kRWordBox + kRTileBytes));
+                    for (int j = 0; j < nw; ++j)
+                        tma_load_3d(st + j * kRWordBox, &xmap, kb * kRSlice, (int)(32 * (wt + j)), layer,
+                                    &full[s]);
+                    tma_load_3d(st + 2 * kRTileBytes, &wmap, kb * kRSlice, 0, layer, &full[s]);
                 }
             }
             // every issued load lands before the CTA may exit
@@ -137,25 +163,29 @@ router_sig_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constan
                                    ((uint32_t)(kRTileM / 16) << 24);
             const uint32_t ring_u32 = smem_u32(ring);
             int g = 0, i = 0;
-            for (int m = blockIdx.x; m < a.ntiles && !*s_abort; m += gridDim.x, ++i) {
+            for (int64_t wt = wb, nw = 0; wt < we && !*s_abort; wt += nw, ++i) {
+                nw = next_tile_words(we - wt);
                 const int buf = i & 1;
+                const int halves = nw > 4 ? 2 : 1;  // the second MMA tile has words
                 if (i >= 2 && !mbar_wait(&acc_free[buf], (uint32_t)((i >> 1) - 1) & 1u, a.status)) {
                     *s_abort = 1;
                     break;
                 }
                 tc_fence_after();
-                const uint32_t d_tmem = tmem + (uint32_t)(buf * kRE);
                 for (int kb = 0; kb < nkb; ++kb, ++g) {
                     const int s = g % kRStages;
                     if (!mbar_wait(&full[s], (uint32_t)(g / kRStages) & 1u, a.status)) *s_abort = 1;
                     if (*s_abort) break;
                     tc_fence_after();
                     const uint32_t sa = ring_u32 + (uint32_t)(s * kRStageBytes);
+                    for (int h = 0; h < halves; ++h) {
+                        const uint32_t d_tmem = tmem + (uint32_t)((2 * buf + h) * kRE);
 #pragma unroll
-                    for (int kk = 0; kk < kRSlice / 16; ++kk)
-                        umma_f16(d_tmem, umma_desc_sw128(sa + kk * 32),
-                                 umma_desc_sw128(sa + kRBoxBytes + kk * 32), idesc,
-                                 (kb > 0 || kk > 0) ? 1u : 0u);
+                        for (int kk = 0; kk < kRSlice / 16; ++kk)
+                            umma_f16(d_tmem, umma_desc_sw128(sa + h * kRTileBytes + kk * 32),
+                                     umma_desc_sw128(sa + 2 * kRTileBytes + kk * 32), idesc,
+                                     (kb > 0 || kk > 0) ? 1u : 0u);
+                    }
                     umma_commit(&empty[s]);  // the stage is free once these MMAs are done
                 }
                 if (*s_abort) break;
@@ -173,7 +203,8 @@ router_sig_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constan
 #pragma unroll
         for (int r = 0; r < kRE / 32; ++r) cnt[r] = 0u;
         int i = 0;
-        for (int m = blockIdx.x; m < a.ntiles; m += gridDim.x, ++i) {
+        for (int64_t wt = wb, nw = 0; wt < we; wt += nw, ++i) {
+            nw = next_tile_words(we - wt);
             const int buf = i & 1;
             const bool ok = !*s_abort && mbar_wait(&acc_full[buf], (uint32_t)(i >> 1) & 1u, a.status);
             if (!__all_sync(kFull, ok)) {  // leave together: the warp collectives below
@@ -181,64 +212,62 @@ router_sig_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constan
                 break;
             }
             tc_fence_after();
-            // this warp's staging tile is free once its previous stores have read it
-            if (lane == 0) bulk_wait_read<0>();
-            __syncwarp();
-            const uint32_t tl = tmem + (uint32_t)(buf * kRE) + ((uint32_t)(quarter * 32) << 16);
+            for (int h = 0; h < 2; ++h) {
+                const int64_t w = wt + 4 * h + quarter;  // this warp's word of tile h
+                const bool mine = 4 * h + quarter < nw;
+                if (mine) {
+                    // the staging tile is free once the previous stores have read it
+                    if (lane == 0) bulk_wait_read<0>();
+                    __syncwarp();
+                    const uint32_t tl =
+                        tmem + (uint32_t)((2 * buf + h) * kRE) + ((uint32_t)(quarter * 32) << 16);
 #pragma unroll
-            for (int b = 0; b < kRE / 32; ++b) {
-                uint32_t v[32];
-                tmem_ld32(tl + 32 * b, v);
-                tmem_wait_ld();
+                    for (int b = 0; b < kRE / 32; ++b) {
+                        uint32_t v[32];
+                        tmem_ld32(tl + 32 * b, v);
+                        tmem_wait_ld();
 #pragma unroll
-                for (int c = 0; c < 8; ++c)
-                    *reinterpret_cast<uint4 *>(chunk_ptr(tp, 8 * b + c, lane)) =
-                        make_uint4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
-            }
-            // the accumulator may be overwritten by the tile after next
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&acc_free[buf]);
-            // the logits of these 32 tokens go out (rows past T are clipped by the map)
-            fence_proxy_async_smem();
-            __syncwarp();
-            const int row0 = m * kRTileM + 32 * quarter;
-            if (lane == 0 && row0 < a.T) {
+                        for (int c = 0; c < 8; ++c)
+                            *reinterpret_cast<uint4 *>(chunk_ptr(tp, 8 * b + c, lane)) =
+                                make_uint4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+                    }
+                }
+                if (h == 1) {  // both accumulators of the pair have been read
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&acc_free[buf]);
+                }
+                if (!mine) continue;
+                // the logits of these 32 tokens go out while the selection reads them
+                fence_proxy_async_smem();
+                __syncwarp();
+                const int row0 = (int)(32 * w);
+                if (lane == 0) {
 #pragma unroll
-                for (int b = 0; b < kRE / 32; ++b) tma_store_3d(&zmap, tp + b * 4096, 32 * b, row0, layer);
-                bulk_commit_group();
-                bulk_wait_read<0>();  // the selection below overwrites the tile
-            }
-            __syncwarp();
-            const int64_t t = (int64_t)row0 + lane;
-            const bool valid = t < a.T;
-            int sel[K];
-            float val[K];
-            select_topk<kRE, K>(tp, lane, sel, val);
-            if (a.idx && valid) store_idx<K>(a.idx + ((int64_t)layer * a.T + t) * K, sel);
-            if (valid) cooc_add<K>(s_cooc, s_rowoff, sel);
-            const int64_t w = (int64_t)row0 / 32;
-            if (w < a.W)
+                    for (int b = 0; b < kRE / 32; ++b)
+                        tma_store_3d(&zmap, tp + b * 4096, 32 * b, row0, layer);
+                    bulk_commit_group();
+                }
+                const int64_t t = (int64_t)row0 + lane;
+                const bool valid = t < a.T;
+                int sel[K];
+                float val[K];
+                select_topk<kRE, K, true>(tp, lane, sel, val);
+                if (a.idx && valid) store_idx<K>(a.idx + ((int64_t)layer * a.T + t) * K, sel);
+                if (valid) cooc_add<K>(tri, s_rowoff, sel);
                 emit_words<kRE, K, true>(sel, valid, lane, a.bits + (int64_t)layer * kRE * a.W + w, a.W,
                                          cnt);
+            }
         }
         if (lane == 0) bulk_wait_all<0>();  // the last stores are complete before exit
-        // counts n_a on the triangle's diagonal
+        // counts n_a: on the triangle's diagonal and into the problem's totals
 #pragma unroll
         for (int r = 0; r < kRE / 32; ++r)
-            if (cnt[r]) atomicAdd(&s_cooc[s_rowoff[32 * r + lane] + 32 * r + lane], cnt[r]);
-        // all epilogue warps have counted: store this CTA's triangle for the
-        // reduction kernel and add its counts to the problem's totals
-        asm volatile("bar.sync 1, %0;" ::"n"(kREpiWarps * 32) : "memory");
-        const int et = threadIdx.x - 64;
-        uint4 *dst = reinterpret_cast<uint4 *>(a.cooc + ((size_t)layer * gridDim.x + blockIdx.x) *
-                                                            (size_t)RC::kCoocWords);
-        const uint4 *src = reinterpret_cast<const uint4 *>(s_cooc);
-        for (int q = et; q < RC::kCoocWords / 4; q += kREpiWarps * 32) dst[q] = src[q];
-        for (int e = et; e < kRE; e += kREpiWarps * 32) {
-            const uint32_t ne = s_cooc[s_rowoff[e] + e];
-            if (ne) atomicAdd(&a.counts[layer * kRE + e], (int)ne);
-        }
+            if (cnt[r]) {
+                const int e = 32 * r + lane;
+                atomicAdd(&tri[s_rowoff[e] + e], cnt[r]);
+                atomicAdd(&a.counts[layer * kRE + e], (int)cnt[r]);
+            }
     }
     tc_fence_before();
     __syncthreads();
@@ -293,8 +322,7 @@ int router_ctas_per_problem(const Problem &p) {
     int sms = sm_count_router();
     if (sms > kMaxSigCtas) sms = kMaxSigCtas;
     int64_t gx = sms / p.L;
-    const int64_t ntiles = (p.T + kRTileM - 1) / kRTileM;
-    if (gx > ntiles) gx = ntiles;
+    if (gx > p.W) gx = p.W;
     if (gx < 1) gx = 1;
     return (int)gx;
 }
@@ -304,7 +332,7 @@ cudaError_t launch_router_signatures(const void *X, const void *Wr, int H, float
                                      uint32_t *cooc, const ZeroSpans &zero, int *status,
                                      cudaStream_t s) {
     CUtensorMap xm, wm, zm;
-    if (!encode_tensor_map_3d_bf16(&xm, X, (uint64_t)p.L, (uint64_t)p.T, (uint64_t)H, kRSlice, kRTileM) ||
+    if (!encode_tensor_map_3d_bf16(&xm, X, (uint64_t)p.L, (uint64_t)p.T, (uint64_t)H, kRSlice, 32) ||
         !encode_tensor_map_3d_bf16(&wm, Wr, (uint64_t)p.L, (uint64_t)kRE, (uint64_t)H, kRSlice, kRE) ||
         !encode_tensor_map_3d_f32(&zm, logits, (uint64_t)p.L, (uint64_t)p.T, (uint64_t)kRE, 32))
         return cudaErrorInvalidValue;
@@ -312,7 +340,6 @@ cudaError_t launch_router_signatures(const void *X, const void *Wr, int H, float
     a.T = p.T;
     a.W = p.W;
     a.H = H;
-    a.ntiles = (int)((p.T + kRTileM - 1) / kRTileM);
     a.bits = bits;
     a.idx = idx;
     a.cooc = cooc;

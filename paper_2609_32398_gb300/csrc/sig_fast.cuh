@@ -126,10 +126,15 @@ __device__ __forceinline__ void store_route(const RouteOut &r, int64_t off, cons
 // (lowest index among equal values), overwritten with -inf in the tile, and
 // the group maximum recomputed.  sel: the chosen experts in selection order;
 // val: their logits.
-template <int E, int K>
+// kMask: chosen experts are excluded through a per-lane bit mask instead of
+// -inf writes, so the tile is only read (it may be in flight to HBM meanwhile).
+template <int E, int K, bool kMask = false>
 __device__ __forceinline__ void select_topk(unsigned char *tp, int lane, int (&sel)[K],
                                             float (&val)[K]) {
     constexpr int GS = SigCfg<E>::GS, NG = SigCfg<E>::NG, GS4 = GS / 4;
+    uint32_t chosen[E / 32];
+#pragma unroll
+    for (int r = 0; r < E / 32; ++r) chosen[r] = 0u;
     float g[NG];
 #pragma unroll
     for (int gi = 0; gi < NG; ++gi) {
@@ -171,6 +176,14 @@ __device__ __forceinline__ void select_topk(unsigned char *tp, int lane, int (&s
             x[4 * c + 2] = v.z;
             x[4 * c + 3] = v.w;
         }
+        if (kMask) {  // the experts of this group chosen before
+            uint32_t word = 0u;
+#pragma unroll
+            for (int r = 0; r < E / 32; ++r) word = ((bi * GS) >> 5) == r ? chosen[r] : word;
+            const uint32_t gm = (word >> ((bi * GS) & 31)) & ((1u << GS) - 1u);
+#pragma unroll
+            for (int j = 0; j < GS; ++j) x[j] = ((gm >> j) & 1u) ? -INFINITY : x[j];
+        }
         int p = GS - 1;
 #pragma unroll
         for (int j = GS - 1; j >= 0; --j)
@@ -179,7 +192,12 @@ __device__ __forceinline__ void select_topk(unsigned char *tp, int lane, int (&s
 #pragma unroll
         for (int j = 0; j < GS; ++j) m2 = fmaxf(m2, j == p ? -INFINITY : x[j]);
         const int e = bi * GS + p;
-        reinterpret_cast<float *>(chunk_ptr(tp, e >> 2, lane))[e & 3] = -INFINITY;
+        if (kMask) {
+#pragma unroll
+            for (int r = 0; r < E / 32; ++r) chosen[r] |= (e >> 5) == r ? 1u << (e & 31) : 0u;
+        } else {
+            reinterpret_cast<float *>(chunk_ptr(tp, e >> 2, lane))[e & 3] = -INFINITY;
+        }
 #pragma unroll
         for (int gi = 0; gi < NG; ++gi) g[gi] = (gi == bi) ? m2 : g[gi];
         sel[qk] = e;
