@@ -81,10 +81,25 @@ def measured_peaks():
         return None
 
 
-def kernel_source_hash():
+# The sources each timed unit's kernels are compiled from (its launcher and
+# argument checks included); a traffic record holds only while they are
+# unchanged.
+UNIT_SOURCES = {
+    "do_forward_backward": ["sig_fast.cuh", "sig_fast.cu", "cooc_reduce.cu", "loss_mma.cu",
+                            "loss.cu", "tma.cuh", "tma_host.cu", "dol_internal.cuh", "api.cu"],
+    "do_routing": ["sig_fast.cuh", "route.cu", "signatures.cu", "tma.cuh", "tma_host.cu",
+                   "dol_internal.cuh", "api.cu"],
+    "do_router_forward_backward": ["router.cu", "sig_fast.cuh", "cooc_reduce.cu", "loss_mma.cu",
+                                   "loss.cu", "tma.cuh", "tma_host.cu", "dol_internal.cuh",
+                                   "api.cu"],
+}
+
+
+def kernel_source_hash(unit="do_forward_backward"):
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2609_32398_gb300", "csrc")
-    for f in sorted(os.listdir(csrc)):
+    for f in sorted(UNIT_SOURCES[unit]):
+        h.update(f.encode())
         h.update(open(os.path.join(csrc, f), "rb").read())
     return h.hexdigest()[:12]
 
@@ -95,7 +110,7 @@ def profiled_traffic(unit):
     path = os.path.join(ROOT, "profiles", "traffic.md")
     if not os.path.exists(path):
         return None
-    src = kernel_source_hash()
+    src = kernel_source_hash(unit)
     for line in open(path):
         m = re.match(r"\|\s*([\w.]+)\s*\|\s*([0-9a-f]{12})\s*\|\s*(\d+)\s*\|", line)
         if m and m.group(1) == unit and m.group(2) == src:
@@ -523,6 +538,9 @@ def run_ours(args, rank, world, local):
 
 
 def main():
+    if len(sys.argv) == 3 and sys.argv[1] == "--source-hash":
+        print(kernel_source_hash(sys.argv[2]))
+        return
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=2000)
