@@ -431,6 +431,18 @@ def run_ours(args, rank, world, local):
     st = dl.device_status(rout.workspace)
     if st != 0:
         raise RuntimeError(f"device status after the router runs: {dl.status_string(st)}")
+    # the router's backward (dz -> bf16 in our kernel, dW and dX in cuBLAS)
+    rbw = torch.empty(int(dl.lib().do_router_backward_workspace_size(T, E, ROUTER_HIDDEN, L)),
+                      dtype=torch.uint8, device=dev)
+    for _ in range(3):
+        dl.router_backward(X, Wr, rout.dlogits, workspace=rbw)
+    ra_.record(stream)
+    for _ in range(router_reps):
+        dl.router_backward(X, Wr, rout.dlogits, workspace=rbw)
+    rb_.record(stream)
+    torch.cuda.synchronize()
+    router_bwd_ms = ra_.elapsed_time(rb_) / router_reps
+    del rbw
     for _ in range(3):
         torch.matmul(X[0], Wr[0].T)
     ra_.record(stream)
@@ -530,6 +542,11 @@ def run_ours(args, rank, world, local):
                              "traffic": profiled_traffic("do_router_forward_backward")},
                 "context_unfused_us": {"cublas_bf16_matmul": cublas_ms * 1e3,
                                        "do_forward_backward": plain_ms * 1e3},
+                "backward": {"entry": "do_router_backward (dz rounded to bf16 by our kernel; dW "
+                                      "fp32 and dX bf16 by cuBLAS)",
+                             "us_per_call": router_bwd_ms * 1e3,
+                             "bytes": 2 * T * L * ROUTER_HIDDEN * 2 + 4 * T * E * L + 4 * T * E * L
+                             + 2 * E * ROUTER_HIDDEN * L + 4 * E * ROUTER_HIDDEN * L},
                 "reps": router_reps},
             "clocks": clocks, "e2e": e2e, "gpu_launches": KERNELS_PER_STEP * args.steps,
             "cpu_baseline": cpu,

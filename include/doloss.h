@@ -179,6 +179,26 @@ do_status do_router_forward_backward(const void *X, const void *Wr, int64_t T, i
                                      float *loss, int64_t *origin_do, float *dlogits,
                                      void *workspace, size_t workspace_bytes, void *stream);
 
+/* Backward of the router's linear map for the gradient dz = dlogits
+ * ([L][T][E] fp32, as written by do_router_forward_backward):
+ *   dW [L][E][H] fp32,  dW[l][e][h] = sum_t dz[l][t][e] X[l][t][h]
+ *   dX [L][T][H] bf16,  dX[l][t][h] = sum_e dz[l][t][e] W[l][e][h]  (may be NULL)
+ * X, W bf16 as in do_router_forward_backward; all arrays 16-byte aligned.
+ * dz is rounded to bf16 (nearest even) by the library and both products run
+ * in cuBLAS (bf16 inputs, fp32 accumulation): plain matrix products with the
+ * reduction index outermost in memory.  cuBLAS is opened at run time; where
+ * it cannot be, the call returns DO_ERR_UNSUPPORTED.  Unlike the other entry
+ * points this one keeps state: the first call on a device creates a cuBLAS
+ * handle for it, and calls are serialised on a lock.  workspace:
+ * do_router_backward_workspace_size bytes of device memory, 256-byte
+ * aligned (the bf16 copy of dz and cuBLAS's workspace).  T <= INT32_MAX and
+ * E H <= INT32_MAX.  Asynchronous on `stream`. */
+do_status do_router_backward(const void *X, const void *Wr, const float *dlogits, int64_t T,
+                             int32_t H, int32_t E, int32_t L, float *dW, void *dX,
+                             void *workspace, size_t workspace_bytes, void *stream);
+
+size_t do_router_backward_workspace_size(int64_t T, int32_t E, int32_t H, int32_t L);
+
 /* Device workspace, in bytes, that do_loss_fwd_bwd and do_forward_backward
  * need for these sizes (0 if the sizes are invalid). */
 size_t do_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L);

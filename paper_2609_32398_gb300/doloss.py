@@ -44,6 +44,9 @@ EXPORTS = {
     "do_forward_backward_routed": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p", "p",
                                     "p", "p", "p", "p", "p", "p", "p", "p", "p", "sz", "p"], "i32"),
     "do_maxvio": (["p", "p", "i32", "i32", "i32", "p", "p", "p", "p"], "i32"),
+    "do_router_backward": (["p", "p", "p", "i64", "i32", "i32", "i32", "p", "p", "p", "sz", "p"],
+                           "i32"),
+    "do_router_backward_workspace_size": (["i64", "i32", "i32", "i32"], "sz"),
     "do_router_forward_backward": (["p", "p", "i64", "i32", "i32", "i32", "i32", "i32", "f32", "p",
                                     "p", "p", "p", "p", "p", "p", "p", "sz", "p"], "i32"),
     "do_rem_allocate": (["p", "p", "p", "i32", "i32", "i32", "p", "p", "p", "p", "p", "p"], "i32"),
@@ -291,6 +294,30 @@ def router_forward_backward(X: torch.Tensor, Wr: torch.Tensor, k, gate=GATE_SIGM
         out.origin_do.data_ptr(), _ptr(out.dlogits), out.workspace.data_ptr(),
         out.workspace.numel(), _stream(X)))
     return logits, out
+
+
+def router_backward(X: torch.Tensor, Wr: torch.Tensor, dlogits: torch.Tensor, with_dx=True,
+                    workspace: torch.Tensor | None = None):
+    """do_router_backward: dW [L,E,H] fp32 and dX [L,T,H] bf16 (or None) of the
+    router's linear map for dlogits [L,T,E] fp32."""
+    if X.dim() == 2:
+        X = X.unsqueeze(0)
+    if Wr.dim() == 2:
+        Wr = Wr.unsqueeze(0)
+    dz = _as3d(dlogits)
+    L, T, H = X.shape
+    E = Wr.shape[1]
+    if dz.shape != (L, T, E) or Wr.shape != (L, E, H):
+        raise ValueError("shapes must be X [L,T,H], Wr [L,E,H], dlogits [L,T,E]")
+    dW = torch.empty(L, E, H, dtype=torch.float32, device=X.device)
+    dX = torch.empty(L, T, H, dtype=torch.bfloat16, device=X.device) if with_dx else None
+    if workspace is None:
+        workspace = torch.empty(int(lib().do_router_backward_workspace_size(T, E, H, L)),
+                                dtype=torch.uint8, device=X.device)
+    _check("do_router_backward", lib().do_router_backward(
+        X.data_ptr(), Wr.data_ptr(), dz.data_ptr(), T, H, E, L, dW.data_ptr(), _ptr(dX),
+        workspace.data_ptr(), workspace.numel(), _stream(X)))
+    return dW, dX
 
 
 def maxvio(counts: torch.Tensor, expert_rank: torch.Tensor, R: int, with_rank_loads=False,

@@ -122,3 +122,17 @@ def test_router_entry_point_validates_on_the_host(dl):
     assert lib.do_router_forward_backward(*args(fake, 1024, 256, 64, 8)) == UNS   # E != 128
     assert lib.do_router_forward_backward(*args(fake, 1024, 96, 128, 8)) == UNS   # H % 64
     assert lib.do_router_forward_backward(*args(fake, 1024, 256, 128, 3)) == UNS  # k
+
+
+def test_router_backward_validates_on_the_host(dl):
+    lib = dl.lib()
+    fake = ctypes.c_void_p(0x10000)
+    odd = ctypes.c_void_p(0x10004)
+    INV, WS = 1, 6
+    big = 1 << 34
+    assert lib.do_router_backward_workspace_size(0, 128, 64, 1) == 0
+    assert lib.do_router_backward_workspace_size(100, 128, 64, 1) >= 2 * 100 * 128
+    assert lib.do_router_backward(None, fake, fake, 64, 64, 128, 1, fake, None, fake, big, None) == INV
+    assert lib.do_router_backward(fake, fake, fake, 64, 64, 128, 1, None, None, fake, big, None) == INV
+    assert lib.do_router_backward(odd, fake, fake, 64, 64, 128, 1, fake, None, fake, big, None) == INV
+    assert lib.do_router_backward(fake, fake, fake, 64, 64, 128, 1, fake, None, fake, 64, None) == WS

@@ -95,3 +95,51 @@ def test_router_path_is_reproducible(dl):
     assert torch.equal(a_logits, b_logits)
     for name in ("bits", "D", "loss", "dlogits"):
         assert torch.equal(getattr(a, name), getattr(b, name)), name
+
+
+def check_router_grads(dW, dX, X, W, dz, cols=None, rows=None):
+    """dW [E,H] fp32 and dX [T,H] bf16 against the oracle's fp64 gradients of the
+    same bf16 X, W and the fp32 dz.  dz is rounded to bf16 (relative error at
+    most 2^-9) and the products accumulate in fp32: per element the error is
+    below (2^-8 + 2 n 2^-24) times the sum of |terms|, n the reduction length;
+    dX is also rounded to bf16 on output (2^-8 of its value)."""
+    T, H = X.shape
+    E = W.shape[0]
+    cols = np.arange(H) if cols is None else cols
+    rows = np.arange(T) if rows is None else rows
+    Xb, Wb = bits16(X), bits16(W)
+    dzd = dz.double().cpu().numpy()
+    Xs = np.ascontiguousarray(Xb[:, cols])
+    Ws = np.ascontiguousarray(Wb[:, cols])
+    dW_ref = oracle.router_grad(Xs, Ws, dzd)
+    absW = np.abs(dzd).T @ np.abs(oracle.bf16_to_double(Xs))
+    got = dW[:, cols].double().cpu().numpy()
+    assert (np.abs(got - dW_ref) <= (2.0 ** -8 + 2 * T * U32) * absW + 1e-30).all()
+    if dX is not None:
+        Xr = np.ascontiguousarray(Xb[rows])
+        _, dX_ref = oracle.router_grad(Xr, Wb, np.ascontiguousarray(dzd[rows]), with_dx=True)
+        absX = np.abs(dzd[rows]) @ np.abs(oracle.bf16_to_double(Wb))
+        gx = dX[rows].double().cpu().numpy()
+        tol = 2.0 ** -8 * np.abs(dX_ref) + (2.0 ** -8 + 2 * E * U32) * absX + 1e-30
+        assert (np.abs(gx - dX_ref) <= tol).all()
+
+
+@pytest.mark.parametrize("T,H,L", [(4096 + 33, 256, 2), (300, 64, 1)])
+def test_router_backward_matches_oracle(dl, T, H, L):
+    X, W = workloads.router_inputs(T, H, 128, L, seed=T + 3 * H, device="cuda")
+    logits, out = dl.router_forward_backward(X, W, 8, 0, grad_scale=1000.0)
+    assert dl.device_status(out.workspace) == 0
+    dW, dX = dl.router_backward(X, W, out.dlogits)
+    for l in range(L):
+        check_router_grads(dW[l], dX[l], X[l], W[l], out.dlogits[l])
+
+
+def test_router_backward_full_size(dl):
+    T, H = 65536, 2048
+    X, W = workloads.router_inputs(T, H, 128, 1, seed=2, device="cuda")
+    _, out = dl.router_forward_backward(X, W, 8, 0, grad_scale=1000.0)
+    dW, dX = dl.router_backward(X, W, out.dlogits)
+    rng = np.random.default_rng(1)
+    check_router_grads(dW[0], dX[0], X[0], W[0], out.dlogits[0],
+                       cols=np.sort(rng.choice(H, 48, replace=False)),
+                       rows=np.sort(rng.choice(T, 256, replace=False)))
