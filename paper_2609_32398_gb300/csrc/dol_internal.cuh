@@ -6,6 +6,8 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include <atomic>
+
 namespace dol {
 
 constexpr unsigned kFull = 0xffffffffu;
@@ -35,6 +37,22 @@ struct RouteOut {
     float *combine;
     int gate;  // 0 sigmoid-norm, 1 softmax
 };
+
+// Raises kernel Kern's dynamic shared-memory limit to `bytes` on the current
+// device.  The attribute belongs to the device's context, so it is set once
+// per device (devices 0..63), not once per process.
+template <auto Kern>
+inline cudaError_t ensure_smem_limit(size_t bytes) {
+    static std::atomic<unsigned long long> done{0ull};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const unsigned long long bit = dev < 64 ? 1ull << dev : 0ull;
+    if (bit && (done.load() & bit)) return cudaSuccess;
+    e = cudaFuncSetAttribute(Kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    if (e == cudaSuccess) done.fetch_or(bit);
+    return e;
+}
 
 // Up to three int ranges that a kernel clears for the kernels after it.
 struct ZeroSpans {

@@ -380,16 +380,9 @@ idx_from_bits_kernel(const uint32_t *__restrict__ bits, int64_t T, int64_t W, in
 template <int E, int K, bool kRFromCounts>
 cudaError_t run_loss_fast(const LossArgs &args, int gate, int P, const Problem &p, cudaStream_t s) {
     const size_t smem = sizeof(int) * E * E;
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(loss_fast_kernel<E, K, 0, kRFromCounts>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(loss_fast_kernel<E, K, 1, kRFromCounts>,
-                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+    cudaError_t e = ensure_smem_limit<loss_fast_kernel<E, K, 0, kRFromCounts>>(smem);
+    if (e == cudaSuccess) e = ensure_smem_limit<loss_fast_kernel<E, K, 1, kRFromCounts>>(smem);
+    if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)P, (unsigned)p.L);
     cfg.blockDim = dim3(kLossFastThreads);

@@ -494,13 +494,8 @@ int sms_now() {
 template <int K>
 cudaError_t run_mma(const CUtensorMap &zmap, const CUtensorMap &dzmap, const MmaArgs &args, int gx,
                     int L, cudaStream_t s) {
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(loss_mma_kernel<K>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMma);
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+    cudaError_t e = ensure_smem_limit<loss_mma_kernel<K>>(kSmemMma);
+    if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)gx, (unsigned)L);
     cfg.blockDim = dim3(kThreads);

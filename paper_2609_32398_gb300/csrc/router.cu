@@ -282,13 +282,8 @@ template <int K>
 cudaError_t run_router(const CUtensorMap &xm, const CUtensorMap &wm, const CUtensorMap &zm,
                        const RouterArgs &a, int ctas, int L, cudaStream_t s) {
     auto kern = router_sig_kernel<K>;
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)kRSmem);
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+    cudaError_t e = ensure_smem_limit<router_sig_kernel<K>>(kRSmem);
+    if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)ctas, (unsigned)L);
     cfg.blockDim = dim3(kRThreads);

@@ -416,13 +416,8 @@ cudaError_t run_fast(const CUtensorMap &map, const Problem &p, uint32_t *bits, i
                      const RouteOut &route, cudaStream_t s) {
     using C = SigCfg<E>;
     auto kern = sig_fast_kernel<E, K, kCounts, kCooc, kRoute>;
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)C::kSmem);
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+    cudaError_t e = ensure_smem_limit<sig_fast_kernel<E, K, kCounts, kCooc, kRoute>>(C::kSmem);
+    if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)sig_fast_ctas_per_problem(p), (unsigned)p.L);
     cfg.blockDim = dim3(kFastThreads);
