@@ -150,8 +150,9 @@ size_t do_routing_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L);
 /* do_forward_backward that also writes the routing outputs of do_routing
  * (expert_ids, combine required; expert_offsets, dispatch_rows, dispatch_pos
  * may each be NULL) from the same selection pass over the logits, so the
- * logits are read once for both the loss and the dispatch.  Same workspace
- * as do_forward_backward. */
+ * logits are read once for both the loss and the dispatch.  workspace:
+ * do_routed_workspace_size(T, E, k, L) bytes (do_forward_backward's plus the
+ * dispatch scratch), prepared as for do_forward_backward. */
 do_status do_forward_backward_routed(const float *logits, int64_t T, int32_t E, int32_t k,
                                      int32_t L, int32_t gate, float grad_scale, uint32_t *bits,
                                      int32_t *counts, int32_t *D, float *loss, int64_t *origin_do,
@@ -199,9 +200,11 @@ do_status do_router_backward(const void *X, const void *Wr, const float *dlogits
 
 size_t do_router_backward_workspace_size(int64_t T, int32_t E, int32_t H, int32_t L);
 
-/* Device workspace, in bytes, that do_loss_fwd_bwd and do_forward_backward
- * need for these sizes (0 if the sizes are invalid). */
+/* Device workspace, in bytes, that do_loss_fwd_bwd, do_forward_backward and
+ * do_router_forward_backward need for these sizes (0 if the sizes are
+ * invalid); do_forward_backward_routed needs do_routed_workspace_size. */
 size_t do_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L);
+size_t do_routed_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L);
 
 /* Synchronizes `stream`, then reads and clears the device-side status that
  * the previous calls with this workspace recorded: DO_OK, DO_ERR_OVERFLOW or

@@ -93,7 +93,7 @@ size_t routing_bits_bytes(const Problem &p) {
 
 size_t routing_ws_bytes(const Problem &p) {
     return dol::kWsHeader + routing_bits_bytes(p) +
-           round_up(sizeof(int) * (size_t)p.L * p.E * (size_t)dol::route_chunks(p), 256);
+           round_up(sizeof(int) * (size_t)dol::route_scratch_ints(p), 256);
 }
 
 HostBufLayout host_layout(const Problem &p) {
@@ -106,7 +106,7 @@ HostBufLayout host_layout(const Problem &p) {
     b.D = off;      off = round_up(off + sizeof(int32_t) * (size_t)p.L * p.E * p.E, 256);
     b.loss = off;   off = round_up(off + sizeof(float) * (size_t)p.L + sizeof(int), 256);  // + status
     b.dlogits = off; off = round_up(off + sizeof(float) * te, 256);
-    b.ws = off;     off = round_up(off + dol::workspace_bytes(p), 256);
+    b.ws = off;     off = round_up(off + dol::workspace_bytes_plain(p), 256);
     b.total = off;
     return b;
 }
@@ -160,7 +160,7 @@ do_status do_loss_fwd_bwd(const float *logits, const uint32_t *bits, const int32
     if (!aligned(logits, 4) || !aligned(bits, 4) || !aligned(D, 4) || !aligned(loss, 4) ||
         (dlogits && !aligned(dlogits, 4)) || (origin_do && !aligned(origin_do, 8)))
         return DO_ERR_INVALID_ARG;
-    if (!workspace || !aligned(workspace, 256) || workspace_bytes < dol::workspace_bytes(p))
+    if (!workspace || !aligned(workspace, 256) || workspace_bytes < dol::workspace_bytes_plain(p))
         return DO_ERR_WORKSPACE;
     cudaStream_t s = (cudaStream_t)stream;
     if (dol::loss_fast_supported(p, logits, D, dlogits) && aligned(bits, 16)) {
@@ -206,8 +206,8 @@ do_status forward_backward_impl(const float *logits, int64_t T, int32_t E, int32
         (origin_do && !aligned(origin_do, 8)))
         return DO_ERR_INVALID_ARG;
     if (ra && (st = check_route(p, *ra)) != DO_OK) return st;
-    if (!workspace || !aligned(workspace, 256) || workspace_bytes < dol::workspace_bytes(p))
-        return DO_ERR_WORKSPACE;
+    const size_t need = ra ? dol::workspace_bytes(p) : dol::workspace_bytes_plain(p);
+    if (!workspace || !aligned(workspace, 256) || workspace_bytes < need) return DO_ERR_WORKSPACE;
     cudaStream_t s = (cudaStream_t)stream;
     const dol::RouteOut route = {ra ? ra->ids : nullptr, ra ? ra->combine : nullptr, gate};
     const bool fast = dol::signatures_fast_supported(logits, p) &&
@@ -243,6 +243,7 @@ do_status forward_backward_impl(const float *logits, int64_t T, int32_t E, int32
                                                       status, route, s)
                  : dol::launch_signatures_fast(logits, p, bits, n_acc, idx, parts, zero, status, s);
         const int P1 = rin ? dol::router_ctas_per_problem(p) : dol::sig_fast_ctas_per_problem(p);
+        int *rscratch = reinterpret_cast<int *>(ws + w.route_base);
         if (e == cudaSuccess)
             e = dol::launch_cooc_reduce(parts, P1, n_acc, p, D, counts, bimg,
                                         reinterpret_cast<long long *>(origin_do), s);
@@ -257,10 +258,10 @@ do_status forward_backward_impl(const float *logits, int64_t T, int32_t E, int32
                                           reinterpret_cast<double *>(ws + w.partials), done,
                                           status, status_out, s);
         }
-        // the dispatch order needs the final counts: after the loss kernel
+        // the dispatch order (from the signatures and ids alone) follows the loss kernel
         if (e == cudaSuccess && ra)
-            e = dol::launch_route_dispatch(bits, counts, ra->ids, p, ra->offsets, ra->rows,
-                                           ra->pos, reinterpret_cast<int *>(ws + w.route_base), s);
+            e = dol::launch_route_dispatch(bits, ra->ids, p, ra->offsets, ra->rows, ra->pos,
+                                           rscratch, s);
         if (e == cudaSuccess && status_done) *status_done = status_out != nullptr;
         return from_cuda(e);
     }
@@ -271,7 +272,7 @@ do_status forward_backward_impl(const float *logits, int64_t T, int32_t E, int32
                              reinterpret_cast<long long *>(origin_do), dlogits, workspace, s);
     if (e == cudaSuccess && ra)
         e = dol::launch_route_dispatch(
-            bits, counts, ra->ids, p, ra->offsets, ra->rows, ra->pos,
+            bits, ra->ids, p, ra->offsets, ra->rows, ra->pos,
             reinterpret_cast<int *>(static_cast<char *>(workspace) + dol::ws_layout(p).route_base), s);
     return from_cuda(e);
 }
@@ -348,7 +349,7 @@ do_status do_routing(const float *logits, int64_t T, int32_t E, int32_t k, int32
     }
     if (e == cudaSuccess)
         e = dol::launch_route_dispatch(
-            bits, counts, expert_ids, p, expert_offsets, dispatch_rows, dispatch_pos,
+            bits, expert_ids, p, expert_offsets, dispatch_rows, dispatch_pos,
             reinterpret_cast<int *>(ws + dol::kWsHeader + routing_bits_bytes(p)), s);
     return from_cuda(e);
 }
@@ -360,6 +361,12 @@ size_t do_routing_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L) {
 }
 
 size_t do_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L) {
+    Problem p;
+    if (check_sizes(T, E, k, L, &p) != DO_OK) return 0;
+    return dol::workspace_bytes_plain(p);
+}
+
+size_t do_routed_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L) {
     Problem p;
     if (check_sizes(T, E, k, L, &p) != DO_OK) return 0;
     return dol::workspace_bytes(p);
@@ -417,7 +424,7 @@ do_status do_forward_backward_host(const float *h_logits, int64_t T, int32_t E, 
     int *d_status = reinterpret_cast<int *>(d_loss + p.L);
     bool status_done = false;
     st = forward_backward_impl(d_logits, T, E, k, L, gate, grad_scale, d_bits, d_counts, d_D,
-                               d_loss, nullptr, d_dlogits, ws, dol::workspace_bytes(p), stream,
+                               d_loss, nullptr, d_dlogits, ws, dol::workspace_bytes_plain(p), stream,
                                d_status, &status_done);
     if (st != DO_OK) return st;
     if (status_done && !h_dlogits && !h_counts && !h_D) {

@@ -69,8 +69,7 @@ struct ZeroSpans {
 //   n_acc           [L][E] int32, counts summed by the signatures CTAs (kept at
 //                   zero between calls: the loss kernel clears it after use)
 //   bimg            [L][kBImageBytes], the fp16 image of D' (E = 128 only)
-//   route_base      [L][E][route chunks] int32, scratch of the dispatch order
-//                   (inside idx when it fits there: it is used after the loss)
+//   route_base      route_scratch_ints int32, scratch of the dispatch order
 struct WsLayout {
     size_t done, partials, idx, cooc_parts, n_acc, bimg, route_base, total;
     int max_parts;  // partial slots per problem
@@ -80,6 +79,8 @@ constexpr int kMaxSigCtas = 256;
 int max_sig_ctas_per_problem(const Problem &p);
 WsLayout ws_layout(const Problem &p);
 inline size_t workspace_bytes(const Problem &p) { return ws_layout(p).total; }
+// What a call without routing outputs needs: the layout up to the routing scratch.
+inline size_t workspace_bytes_plain(const Problem &p) { return ws_layout(p).route_base; }
 
 // Number of generic loss-kernel CTAs per problem; fixes the partial-sum
 // layout and therefore the reduction order.
@@ -109,13 +110,14 @@ cudaError_t launch_signatures_fast_routed(const float *logits, const Problem &p,
                                           const ZeroSpans &zero, int *status,
                                           const RouteOut &route, cudaStream_t s);
 // Dispatch order of the routed (token, choice) pairs from the signatures and
-// the final counts: offsets [L][E+1], rows [L][T k], pos [L][T][k] (each may
-// be null).  chunk_base: scratch of route_chunks(p) * E * L ints.  Launched as
-// programmatic dependents of the previous kernel.
+// the chosen ids alone: offsets [L][E+1], rows [L][T k], pos [L][T][k] (each
+// may be null).  scratch: route_scratch_ints(p) ints.  Launched as
+// programmatic dependents of the previous kernel on `s`.
 int64_t route_chunks(const Problem &p);
-cudaError_t launch_route_dispatch(const uint32_t *bits, const int *counts, const int *ids,
-                                  const Problem &p, int *offsets, int *rows, int *pos,
-                                  int *chunk_base, cudaStream_t s);
+int64_t route_scratch_ints(const Problem &p);
+cudaError_t launch_route_dispatch(const uint32_t *bits, const int *ids, const Problem &p,
+                                  int *offsets, int *rows, int *pos, int *scratch,
+                                  cudaStream_t s);
 // Router-side fusion (E = 128, k in {1,2,4,8}, H a multiple of 64, 16-byte
 // aligned X, W and logits): logits = X W^T on the tensor cores with the
 // fused path's signature step in the epilogue (bits, selected indices,

@@ -248,14 +248,10 @@ WsLayout ws_layout(const Problem &p) {
                                             : 0;
     w.n_acc = up(w.cooc_parts + parts);
     w.bimg = up(w.n_acc + ((fast_k && fast_e) ? sizeof(int) * (size_t)p.L * p.E : 0));
-    const size_t end = up(w.bimg + ((fast_k && p.E == 128) ? (size_t)kBImageBytes * (size_t)p.L : 0));
-    // The dispatch order of a routed call runs after the loss kernel, when the
-    // selected-index bytes are no longer read: its scratch shares their region
-    // where it fits.
-    const size_t route_need = sizeof(int) * (size_t)p.L * p.E * (size_t)route_chunks(p);
-    const size_t idx_bytes = fast_k ? (size_t)p.L * (size_t)p.T * (size_t)p.k : 0;
-    w.route_base = route_need <= idx_bytes ? w.idx : end;
-    w.total = route_need <= idx_bytes ? end : up(end + route_need);
+    // the dispatch order of a routed call may run beside the loss kernel: its
+    // scratch has a region of its own
+    w.route_base = up(w.bimg + ((fast_k && p.E == 128) ? (size_t)kBImageBytes * (size_t)p.L : 0));
+    w.total = up(w.route_base + sizeof(int) * (size_t)route_scratch_ints(p));
     return w;
 }
 

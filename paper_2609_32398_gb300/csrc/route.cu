@@ -22,20 +22,18 @@ constexpr int kScatterThreads = 256;
 constexpr int kMaxChunkWords = 32;
 constexpr int kBatch = 8;  // independent global loads a scatter thread keeps in flight
 
-// Kernel 1, one CTA per (expert e, problem): the offset of e (the counts of
-// the experts before it) and, for every chunk of C = 2^lc signature words,
-// the first row of e's tokens in that chunk:
-//   chunk_base[c] = offsets[e] + (set bits of F_e in chunks 0 .. c-1).
+// Kernel 1, one CTA per (expert e, problem): n_e and, for every chunk of
+// C = 2^lc signature words, the first row of e's tokens in that chunk counted
+// from the start of e's rows:
+//   chunk_base[c] = set bits of F_e in chunks 0 .. c-1,   totals[e] = n_e.
 // A thread sums its chunk's population counts; a block-wide exclusive scan
 // over the chunks of a pass (kScanThreads chunks) and the running total of
-// the passes before it give the bases.  The first pass's loads are issued
-// together with those of the counts, before any barrier.
+// the passes before it give the bases.  Only the signatures are read, so the
+// dispatch order can be built as soon as the selection is done.
 __global__ void __launch_bounds__(kScanThreads)
-route_scan_kernel(const uint32_t *__restrict__ bits, const int *__restrict__ counts, int E,
-                  int64_t W, int lc, int64_t nchunks, int *__restrict__ offsets,
-                  int *__restrict__ chunk_base) {
+route_scan_kernel(const uint32_t *__restrict__ bits, int E, int64_t W, int lc, int64_t nchunks,
+                  int *__restrict__ chunk_base, int *__restrict__ totals) {
     __shared__ int s_warp[kScanWarps];
-    __shared__ int s_base;
     const int e = blockIdx.x, layer = blockIdx.y;
     const int tid = threadIdx.x, lane = tid & 31, wp = tid >> 5;
     const int C = 1 << lc;
@@ -52,33 +50,14 @@ route_scan_kernel(const uint32_t *__restrict__ bits, const int *__restrict__ cou
         for (int j = 0; j < kMaxChunkWords; ++j) n += __popc(v[j]);
         return n;
     };
-    // the signatures and counts come from the kernels before this one
+    // the signatures come from the kernel before this one
     pdl_wait();
     pdl_trigger();
-    const int *cl = counts + (size_t)layer * E;
-    int part = 0;
-    for (int i = tid; i < e; i += kScanThreads) part += __ldg(cl + i);
-    int n = chunk_base ? chunk_count(tid) : 0;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(kFull, part, o);
-    if (lane == 0) s_warp[wp] = part;
-    __syncthreads();
-    if (tid == 0) {
-        int b = 0;
-        for (int q = 0; q < kScanWarps; ++q) b += s_warp[q];
-        s_base = b;
-        if (offsets) {
-            offsets[(size_t)layer * (E + 1) + e] = b;
-            if (e == E - 1) offsets[(size_t)layer * (E + 1) + E] = b + cl[e];
-        }
-    }
-    __syncthreads();
-    if (!chunk_base) return;
-    int run = s_base;
+    int run = 0;
     int *cb = chunk_base + ((size_t)layer * E + e) * nchunks;
     for (int64_t c0 = 0; c0 < nchunks; c0 += kScanThreads) {
         const int64_t c = c0 + tid;
-        if (c0 > 0) n = chunk_count(c);
+        const int n = chunk_count(c);
         int x = n;  // inclusive scan inside the warp
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
@@ -98,6 +77,7 @@ route_scan_kernel(const uint32_t *__restrict__ bits, const int *__restrict__ cou
         if (c < nchunks) cb[c] = run + before + x - n;
         run += total;
     }
+    if (tid == 0) totals[(size_t)layer * E + e] = run;
 }
 
 // Kernel 2, one CTA per (chunk of C = 2^lc signature words = 32 C tokens,
@@ -113,8 +93,9 @@ route_scan_kernel(const uint32_t *__restrict__ bits, const int *__restrict__ cou
 // is a power of two (the pair index is then split by a shift), else -1.
 __global__ void __launch_bounds__(kScatterThreads)
 route_scatter_kernel(const uint32_t *__restrict__ bits, const int *__restrict__ ids,
-                     const int *__restrict__ chunk_base, int T, int E, int k, int lk, int64_t W,
-                     int lc, int64_t nchunks, int *__restrict__ rows, int *__restrict__ pos) {
+                     const int *__restrict__ chunk_base, const int *__restrict__ totals, int T,
+                     int E, int k, int lk, int64_t W, int lc, int64_t nchunks,
+                     int *__restrict__ offsets, int *__restrict__ rows, int *__restrict__ pos) {
     extern __shared__ int smem_i[];
     const int C = 1 << lc, EC = E << lc;
     uint32_t *s_bits = reinterpret_cast<uint32_t *>(smem_i);  // [E][C]
@@ -152,9 +133,48 @@ route_scatter_kernel(const uint32_t *__restrict__ bits, const int *__restrict__ 
             if (i < EC) s_bits[i] = v[u];
         }
     }
-    for (int e = tid; e < E; e += kScatterThreads)
-        s_cb[e] = chunk_base[((size_t)layer * E + e) * nchunks + c];
+    // first row of every expert: an exclusive scan of the totals (E <= 1024,
+    // at most four consecutive experts per thread)
+    {
+        __shared__ int s_wsum[kScatterThreads / 32];
+        const int lane = tid & 31, wp = tid >> 5;
+        const int per = (E + kScatterThreads - 1) / kScatterThreads;
+        const int *tl = totals + (size_t)layer * E;
+        int loc[4], sum = 0;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int e = tid * per + j;
+            const int v = (j < per && e < E) ? __ldg(tl + e) : 0;
+            loc[j] = sum;
+            sum += v;
+        }
+        int x = sum;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(kFull, x, o);
+            if (lane >= o) x += y;
+        }
+        if (lane == 31) s_wsum[wp] = x;
+        __syncthreads();
+        int before = 0, all = 0;
+#pragma unroll
+        for (int q = 0; q < kScatterThreads / 32; ++q) {
+            before += q < wp ? s_wsum[q] : 0;
+            all += s_wsum[q];
+        }
+        const int excl = before + x - sum;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int e = tid * per + j;
+            if (j < per && e < E) {
+                s_cb[e] = excl + loc[j] + chunk_base[((size_t)layer * E + e) * nchunks + c];
+                if (offsets && c == 0) offsets[(size_t)layer * (E + 1) + e] = excl + loc[j];
+            }
+        }
+        if (offsets && c == 0 && tid == 0) offsets[(size_t)layer * (E + 1) + E] = all;
+    }
     __syncthreads();
+    if (!rows && !pos) return;
     for (int e = tid; e < E; e += kScatterThreads) {
         int acc = 0;
         for (int j = 0; j < C; ++j) {
@@ -235,15 +255,16 @@ int64_t route_chunks(const Problem &p) {
     return (p.W + C - 1) / C;
 }
 
-cudaError_t launch_route_dispatch(const uint32_t *bits, const int *counts, const int *ids,
-                                  const Problem &p, int *offsets, int *rows, int *pos,
-                                  int *chunk_base, cudaStream_t s) {
+cudaError_t launch_route_dispatch(const uint32_t *bits, const int *ids, const Problem &p,
+                                  int *offsets, int *rows, int *pos, int *scratch,
+                                  cudaStream_t s) {
     if (!offsets && !rows && !pos) return cudaSuccess;
     const int C = route_chunk_words(p);
     int lc = 0;
     while ((1 << lc) < C) ++lc;
     const int64_t nchunks = route_chunks(p);
-    int *cb = (rows || pos) ? chunk_base : nullptr;
+    int *chunk_base = scratch;
+    int *totals = scratch + (size_t)p.L * p.E * nchunks;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
@@ -253,15 +274,18 @@ cudaError_t launch_route_dispatch(const uint32_t *bits, const int *counts, const
     cfg.stream = s;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, route_scan_kernel, bits, counts, p.E, p.W, lc,
-                                       nchunks, offsets, cb);
-    if (e != cudaSuccess || !cb) return e;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, route_scan_kernel, bits, p.E, p.W, lc, nchunks,
+                                       chunk_base, totals);
+    if (e != cudaSuccess) return e;
     cfg.gridDim = dim3((unsigned)nchunks, (unsigned)p.L);
     cfg.blockDim = dim3(kScatterThreads);
     cfg.dynamicSmemBytes = sizeof(int) * (size_t)(2 * p.E * C + p.E);
     const int lk = (p.k & (p.k - 1)) == 0 ? __builtin_ctz((unsigned)p.k) : -1;
-    return cudaLaunchKernelEx(&cfg, route_scatter_kernel, bits, ids, (const int *)cb, (int)p.T,
-                              p.E, p.k, lk, p.W, lc, nchunks, rows, pos);
+    return cudaLaunchKernelEx(&cfg, route_scatter_kernel, bits, ids, (const int *)chunk_base,
+                              (const int *)totals, (int)p.T, p.E, p.k, lk, p.W, lc, nchunks,
+                              offsets, rows, pos);
 }
+
+int64_t route_scratch_ints(const Problem &p) { return (int64_t)p.L * p.E * (route_chunks(p) + 1); }
 
 }  // namespace dol

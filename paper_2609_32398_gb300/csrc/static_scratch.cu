@@ -56,12 +56,18 @@ extern "C" do_status do_forward_backward_static(const float *logits, int64_t T, 
                                                 float *dlogits, int32_t *status_flags,
                                                 void *stream) {
     // the sizes are checked by do_workspace_size (0 = invalid) before anything else
-    const size_t need = do_workspace_size(T, E, k, L);
-    if (need == 0) {
+    if (do_workspace_size(T, E, k, L) == 0) {
         if (T < 1 || E < 1 || k < 1 || k > E || L < 1) return DO_ERR_INVALID_ARG;
         return DO_ERR_UNSUPPORTED;
     }
-    if (need > DO_STATIC_SCRATCH_BYTES) return DO_ERR_WORKSPACE;
+    dol::Problem p;
+    p.T = T;
+    p.E = E;
+    p.k = k;
+    p.L = L;
+    p.W = (T + 31) / 32;
+    // no routing outputs here: the layout up to the routing scratch
+    if (dol::workspace_bytes_plain(p) > DO_STATIC_SCRATCH_BYTES) return DO_ERR_WORKSPACE;
     if (!logits || !bits || !counts || !D || !loss) return DO_ERR_INVALID_ARG;
     if (status_flags && reinterpret_cast<uintptr_t>(status_flags) % 4 != 0)
         return DO_ERR_INVALID_ARG;
@@ -73,16 +79,11 @@ extern "C" do_status do_forward_backward_static(const float *logits, int64_t T, 
     // counters (the first 256-byte-aligned span) and the counts accumulator
     // (the last span).  The kernels leave them zero after a complete call;
     // clearing them here also recovers from a call that gave up on a wait.
-    dol::Problem p;
-    p.T = T;
-    p.E = E;
-    p.k = k;
-    p.L = L;
-    p.W = (T + 31) / 32;
     const dol::WsLayout w = dol::ws_layout(p);
     char *base = static_cast<char *>(ws);
     if (cudaMemsetAsync(base, 0, w.partials, s) != cudaSuccess) return DO_ERR_CUDA;
-    if (w.total > w.n_acc && cudaMemsetAsync(base + w.n_acc, 0, w.total - w.n_acc, s) != cudaSuccess)
+    if (w.route_base > w.n_acc &&
+        cudaMemsetAsync(base + w.n_acc, 0, w.route_base - w.n_acc, s) != cudaSuccess)
         return DO_ERR_CUDA;
     st = do_forward_backward(logits, T, E, k, L, gate, grad_scale, bits, counts, D, loss, origin_do,
                              dlogits, ws, DO_STATIC_SCRATCH_BYTES, stream);

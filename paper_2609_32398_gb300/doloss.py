@@ -30,6 +30,7 @@ EXPORTS = {
     "do_forward_backward": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p", "p", "p",
                              "p", "p", "p", "sz", "p"], "i32"),
     "do_workspace_size": (["i64", "i32", "i32", "i32"], "sz"),
+    "do_routed_workspace_size": (["i64", "i32", "i32", "i32"], "sz"),
     "do_device_status": (["p", "p"], "i32"),
     "do_forward_backward_host": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p", "p",
                                   "p", "p", "sz", "p"], "i32"),
@@ -115,8 +116,8 @@ def workspace_size(T: int, E: int, k: int, L: int = 1) -> int:
     return int(lib().do_workspace_size(T, E, k, L))
 
 
-def new_workspace(T: int, E: int, k: int, L: int = 1, device="cuda") -> torch.Tensor:
-    n = workspace_size(T, E, k, L)
+def new_workspace(T: int, E: int, k: int, L: int = 1, device="cuda", routed=False) -> torch.Tensor:
+    n = int(lib().do_routed_workspace_size(T, E, k, L)) if routed else workspace_size(T, E, k, L)
     if n == 0:
         raise ValueError("invalid sizes")
     return torch.zeros(n, dtype=torch.uint8, device=device)
@@ -182,7 +183,8 @@ class Buffers:
         self.loss = torch.empty(L, dtype=torch.float32, device=device)
         self.origin_do = torch.empty(L, dtype=torch.int64, device=device)
         self.dlogits = torch.empty(L, T, E, dtype=torch.float32, device=device) if with_grad else None
-        self.workspace = new_workspace(T, E, k, L, device)
+        # large enough for the routed call as well
+        self.workspace = new_workspace(T, E, k, L, device, routed=True)
 
 
 def forward_backward(logits, k, gate=GATE_SIGMOID_NORM, grad_scale=1.0, out: Buffers | None = None,

@@ -84,8 +84,9 @@ def test_routing_entry_points_validate_on_the_host(dl):
     INV, UNS, WS = 1, 2, 6
     big_ws = 1 << 30
     assert dl.lib().do_routing_workspace_size(0, 8, 2, 1) == 0
-    # status word + padding, the signatures [L][E][W], one dispatch chunk base
-    # per expert and problem (W = 32 words is one chunk), each rounded to 256 B
+    # status word + padding, the signatures [L][E][W], and per expert and
+    # problem one dispatch chunk base (W = 32 words is one chunk) and a total,
+    # each region rounded to 256 B
     assert dl.lib().do_routing_workspace_size(1000, 8, 2, 3) == 256 + 4 * 3 * 8 * 32 + 256
     assert lib.do_routing(fake, 64, 8, 2, 1, 0, None, fake, fake, None, None, None, fake, big_ws,
                           None) == INV                                        # no expert_ids
