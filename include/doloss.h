@@ -228,6 +228,21 @@ do_status do_forward_backward_host(const float *h_logits, int64_t T, int32_t E, 
 
 size_t do_host_buffer_size(int64_t T, int32_t E, int32_t k, int32_t L);
 
+/* do_forward_backward_host without the wait, for pipelines that keep the host
+ * link busy: enqueues on `stream` the copy of h_logits to the device, steps
+ * 1-3 and one copy back of the result into h_result (host memory, pinned for
+ * the copies to overlap): bytes [0, 4L) the losses (fp32), bytes [4L, 4L+4)
+ * the int32 device status word of this call (bit 0: a Hamming row sum did
+ * not fit int32; bit 1: a bounded wait ran out; 0: success).  Returns once
+ * the work is enqueued; h_logits must stay unchanged and h_result unread
+ * until `stream` has reached that point.  device_buffer as for
+ * do_forward_backward_host; calls that share one device_buffer must be
+ * ordered on one stream. */
+do_status do_forward_backward_host_async(const float *h_logits, int64_t T, int32_t E, int32_t k,
+                                         int32_t L, int32_t gate, float grad_scale,
+                                         void *h_result, void *device_buffer,
+                                         size_t device_buffer_bytes, void *stream);
+
 /* Largest workspace, in bytes, that do_forward_backward_static can hold. */
 #define DO_STATIC_SCRATCH_BYTES ((size_t)16 << 20)
 

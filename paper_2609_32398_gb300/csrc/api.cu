@@ -460,6 +460,46 @@ do_status do_forward_backward_host(const float *h_logits, int64_t T, int32_t E, 
     return do_device_status(ws, stream);
 }
 
+do_status do_forward_backward_host_async(const float *h_logits, int64_t T, int32_t E, int32_t k,
+                                         int32_t L, int32_t gate, float grad_scale,
+                                         void *h_result, void *device_buffer,
+                                         size_t device_buffer_bytes, void *stream) {
+    NvtxRange nvtx("do_forward_backward_host_async");
+    Problem p;
+    do_status st = check_sizes(T, E, k, L, &p);
+    if (st != DO_OK) return st;
+    if (!h_logits || !h_result || !aligned(h_result, 4)) return DO_ERR_INVALID_ARG;
+    const HostBufLayout b = host_layout(p);
+    if (!device_buffer || !aligned(device_buffer, 256) || device_buffer_bytes < b.total)
+        return DO_ERR_WORKSPACE;
+    char *base = static_cast<char *>(device_buffer);
+    float *d_logits = reinterpret_cast<float *>(base + b.logits);
+    float *d_loss = reinterpret_cast<float *>(base + b.loss);
+    int *d_status = reinterpret_cast<int *>(d_loss + p.L);
+    void *ws = base + b.ws;
+    cudaStream_t s = (cudaStream_t)stream;
+    const size_t te = sizeof(float) * (size_t)p.L * p.T * p.E;
+    // a cleared status word: the result of this call reports this call only
+    cudaError_t e = cudaMemsetAsync(ws, 0, sizeof(int), s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(d_logits, h_logits, te, cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return DO_ERR_CUDA;
+    bool status_done = false;
+    st = forward_backward_impl(d_logits, T, E, k, L, gate, grad_scale,
+                               reinterpret_cast<uint32_t *>(base + b.bits),
+                               reinterpret_cast<int32_t *>(base + b.counts),
+                               reinterpret_cast<int32_t *>(base + b.D), d_loss, nullptr,
+                               reinterpret_cast<float *>(base + b.dlogits), ws,
+                               dol::workspace_bytes_plain(p), stream, d_status, &status_done);
+    if (st != DO_OK) return st;
+    // outside the fused path the status word stays in the workspace: put it
+    // behind the losses, so that one copy returns both
+    if (!status_done) e = cudaMemcpyAsync(d_status, ws, sizeof(int), cudaMemcpyDeviceToDevice, s);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(h_result, d_loss, sizeof(float) * p.L + sizeof(int),
+                            cudaMemcpyDeviceToHost, s);
+    return from_cuda(e);
+}
+
 const char *do_status_string(int32_t status) {
     switch (status) {
         case DO_OK: return "ok";

@@ -35,6 +35,8 @@ EXPORTS = {
     "do_forward_backward_host": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p", "p",
                                   "p", "p", "sz", "p"], "i32"),
     "do_host_buffer_size": (["i64", "i32", "i32", "i32"], "sz"),
+    "do_forward_backward_host_async": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p",
+                                        "sz", "p"], "i32"),
     "do_status_string": (["i32"], "str"),
     "do_selftest_wait_limit": (["p", "p"], "i32"),
     "do_forward_backward_static": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p", "p",
@@ -393,6 +395,33 @@ def forward_backward_host(h_logits: torch.Tensor, k, gate=GATE_SIGMOID_NORM, gra
         _ptr(h_counts), _ptr(h_D), device_buffer.data_ptr(), device_buffer.numel(),
         torch.cuda.current_stream(device_buffer.device).cuda_stream))
     return h_loss
+
+
+def forward_backward_host_async(h_logits: torch.Tensor, k, h_result: torch.Tensor,
+                                device_buffer: torch.Tensor, gate=GATE_SIGMOID_NORM,
+                                grad_scale=1.0, stream: torch.cuda.Stream | None = None):
+    """do_forward_backward_host_async: enqueue the copy in, steps 1-3 and the
+    copy of the losses and the status word into h_result (a pinned CPU tensor
+    of at least 4 (L + 1) bytes) on `stream` (default: the current stream).
+    Read the result with `host_result` once the stream has been synchronized."""
+    z = h_logits.unsqueeze(0) if h_logits.dim() == 2 else h_logits
+    if z.is_cuda or z.dtype != torch.float32 or not z.is_contiguous():
+        raise ValueError("h_logits must be a contiguous CPU float32 tensor")
+    L, T, E = z.shape
+    if h_result.is_cuda or h_result.numel() * h_result.element_size() < 4 * (L + 1):
+        raise ValueError("h_result must be a CPU tensor of at least 4 (L + 1) bytes")
+    st = stream if stream is not None else torch.cuda.current_stream(device_buffer.device)
+    _check("do_forward_backward_host_async", lib().do_forward_backward_host_async(
+        z.data_ptr(), T, E, k, L, gate, grad_scale, h_result.data_ptr(), device_buffer.data_ptr(),
+        device_buffer.numel(), st.cuda_stream))
+
+
+def host_result(h_result: torch.Tensor, L: int):
+    """(losses [L] float32, device status flags int) from an async call's result."""
+    raw = h_result.view(torch.uint8)[: 4 * (L + 1)]
+    loss = raw[: 4 * L].view(torch.float32).clone()
+    flags = int(raw[4 * L: 4 * L + 4].view(torch.int32)[0])
+    return loss, flags
 
 
 def forward_backward_static(logits, k, out: Buffers, gate=GATE_SIGMOID_NORM, grad_scale=1.0,

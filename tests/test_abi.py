@@ -137,3 +137,15 @@ def test_router_backward_validates_on_the_host(dl):
     assert lib.do_router_backward(fake, fake, fake, 64, 64, 128, 1, None, None, fake, big, None) == INV
     assert lib.do_router_backward(odd, fake, fake, 64, 64, 128, 1, fake, None, fake, big, None) == INV
     assert lib.do_router_backward(fake, fake, fake, 64, 64, 128, 1, fake, None, fake, 64, None) == WS
+
+
+def test_async_host_entry_validates_on_the_host(dl):
+    lib = dl.lib()
+    fake = ctypes.c_void_p(0x10000)
+    INV, WS = 1, 6
+    assert lib.do_forward_backward_host_async(fake, 64, 8, 2, 1, 0, 1.0, None, fake, 1 << 30,
+                                              None) == INV
+    assert lib.do_forward_backward_host_async(None, 64, 8, 2, 1, 0, 1.0, fake, fake, 1 << 30,
+                                              None) == INV
+    assert lib.do_forward_backward_host_async(fake, 64, 8, 2, 1, 0, 1.0, fake, fake, 64,
+                                              None) == WS

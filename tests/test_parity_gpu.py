@@ -281,3 +281,23 @@ def test_bounded_wait_reports_timeout_and_context_survives(dl):
     assert dl.device_status(out.workspace) == 0
     ref = oracle.forward_backward(z[0].cpu().numpy(), w.k, w.gate)
     assert np.array_equal(out.D[0].cpu().numpy(), ref["D"])
+
+
+@pytest.mark.parametrize("T,E,k,gate", [(65536, 128, 8, 0), (1000, 33, 3, 1)])
+def test_async_host_entry_matches_the_synchronous_one(dl, T, E, k, gate):
+    """do_forward_backward_host_async: the same loss as the synchronous host
+    entry point (fused and generic paths), with the status word behind it;
+    two calls in flight on two streams and two device buffers."""
+    z = workloads.random_logits(T, E, seed=T + E)[0].contiguous().pin_memory()
+    want = dl.forward_backward_host(z, k, gate).clone()
+    bufs = [torch.zeros(dl.host_buffer_size(T, E, k, 1), dtype=torch.uint8, device="cuda")
+            for _ in range(2)]
+    res = [torch.zeros(8, dtype=torch.int32).pin_memory() for _ in range(2)]
+    streams = [torch.cuda.Stream() for _ in range(2)]
+    for i in range(4):
+        dl.forward_backward_host_async(z, k, res[i % 2], bufs[i % 2], gate, stream=streams[i % 2])
+    torch.cuda.synchronize()
+    for r in res:
+        loss, flags = dl.host_result(r, 1)
+        assert flags == 0
+        assert torch.equal(loss, want)
