@@ -10,6 +10,10 @@
  *   3. the surrogate loss and its gradient to the router logits
  *                                                       (Sec. 3.1.3, Eq. do_loss)
  *   4. Eq. origin_do, the sum of squared distances, as a diagnostic.
+ * and around them: the router's outputs (do_routing), the router's linear map
+ * fused with step 1 and its backward (do_router_forward_backward,
+ * do_router_backward), and the consumers of the counts (do_maxvio,
+ * do_rem_allocate).
  *
  * Notation: E experts (the paper's n), k selected per token (K), T tokens in
  * the signature window (m), L independent problems batched in one call (for
@@ -17,8 +21,11 @@
  *
  * Conventions shared by every entry point:
  *  - Every array argument is a DEVICE pointer owned by the caller, except in
- *    do_forward_backward_host, whose h_* arguments are host pointers.  The
- *    library allocates nothing and keeps no state between calls.
+ *    do_forward_backward_host(_async), whose h_* arguments are host pointers,
+ *    and do_rem_allocate, a host function.  The library allocates nothing and
+ *    keeps no state between calls, with two stated exceptions:
+ *    do_forward_backward_static (a fixed scratch array per device) and
+ *    do_router_backward (a cuBLAS handle per device).
  *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default
  *    stream).  Calls are asynchronous on it, except do_device_status and
  *    do_forward_backward_host, which synchronize it.

@@ -86,7 +86,7 @@ bool route_fast_ok(const RouteArgs *r) {
 }
 
 // Workspace of do_routing: [status word | pad to 256 B | signatures [L][E][W] |
-// dispatch scratch [L][E][route chunks]].
+// dispatch scratch (route_scratch_ints)].
 size_t routing_bits_bytes(const Problem &p) {
     return round_up(sizeof(uint32_t) * (size_t)p.L * p.E * p.W, 256);
 }
