@@ -21,9 +21,14 @@
 //            tiles): the logits go TMEM -> registers -> a swizzled shared-memory
 //            tile (the signature kernel's layout), out to HBM by TMA stores, and
 //            the signature kernel's per-token selection and signature words run
-//            on that tile.  The co-occurrence counts go straight to this CTA's
-//            partial triangle in global memory (L2 reductions): shared memory
-//            is kept for the ring.
+//            on that tile.  The co-occurrence counts go into a shared triangle
+//            of 16-bit counters (two per word: the CTA's range is below 65536
+//            tokens), written out unpacked at the end; for longer ranges they
+//            go straight to the CTA's triangle in global memory as L2
+//            reductions.
+#include <cstdlib>
+#include <cstring>
+
 #include "sig_fast.cuh"
 
 namespace dol {
@@ -45,7 +50,8 @@ using RC = SigCfg<kRE>;
 
 constexpr size_t kROffZ = (size_t)kRStages * kRStageBytes;
 constexpr size_t kROffRowoff = kROffZ + (size_t)kREpiWarps * kRZTileBytes;
-constexpr size_t kROffBars = kROffRowoff + (size_t)kRE * 4;
+constexpr size_t kROffTri = kROffRowoff + (size_t)kRE * 4;          // packed 16-bit counters
+constexpr size_t kROffBars = kROffTri + (size_t)(RC::kCoocWords / 2) * 4;
 constexpr size_t kRNumBars = 2 * kRStages + 4;
 constexpr size_t kROffScal = kROffBars + kRNumBars * 8;
 constexpr size_t kRSmem = kROffScal + 16 + 1024;  // + alignment slack of the base
@@ -53,6 +59,7 @@ constexpr size_t kRSmem = kROffScal + 16 + 1024;  // + alignment slack of the ba
 struct RouterArgs {
     int64_t T, W;
     int H;
+    int packed;  // 1: 16-bit shared counters (no CTA range above 65535 tokens); 0: L2 reductions
     uint32_t *bits;
     uint8_t *idx;
     uint32_t *cooc;
@@ -77,6 +84,7 @@ router_sig_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constan
     unsigned char *ring = smem;
     unsigned char *ztiles = smem + kROffZ;
     int *s_rowoff = reinterpret_cast<int *>(smem + kROffRowoff);
+    uint32_t *s_tri = reinterpret_cast<uint32_t *>(smem + kROffTri);
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kROffBars);
     uint64_t *full = bars, *empty = bars + kRStages;
     uint64_t *acc_full = bars + 2 * kRStages, *acc_free = acc_full + 2;
@@ -95,6 +103,8 @@ router_sig_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constan
     // Shared-memory and TMEM set-up touch no global memory: they overlap the
     // end of the previous kernel on the stream.
     for (int e = threadIdx.x; e < kRE; e += kRThreads) s_rowoff[e] = cooc_row_offset<kRE>(e) - (e & ~3);
+    if (a.packed)
+        for (int i = threadIdx.x; i < RC::kCoocWords / 2; i += kRThreads) s_tri[i] = 0u;
     if (threadIdx.x == 0) {
         for (int s = 0; s < kRStages; ++s) {
             mbar_init(&full[s], 1);
@@ -125,8 +135,7 @@ router_sig_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constan
         for (int64_t i = (int64_t)blockIdx.x * kRThreads + threadIdx.x; i < a.zero.n[z];
              i += (int64_t)gridDim.x * kRThreads)
             a.zero.p[z][i] = 0;
-    {  // the triangle starts at zero; the barrier below orders these stores
-       // before the reductions of the epilogue
+    if (!a.packed) {  // the global triangle starts at zero (ordered by the barrier)
         uint4 *t4 = reinterpret_cast<uint4 *>(tri);
         for (int q = threadIdx.x; q < RC::kCoocWords / 4; q += kRThreads) t4[q] = make_uint4(0u, 0u, 0u, 0u);
     }
@@ -254,7 +263,29 @@ router_sig_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constan
                 float val[K];
                 select_topk<kRE, K, true>(tp, lane, sel, val);
                 if (a.idx && valid) store_idx<K>(a.idx + ((int64_t)layer * a.T + t) * K, sel);
-                if (valid) cooc_add<K>(tri, s_rowoff, sel);
+                if (valid) {  // c_ab += 1 for the pairs a < b, 16-bit halves of shared words
+                    int so[K];
+#pragma unroll
+                    for (int q = 0; q < K; ++q) so[q] = sel[q];
+#pragma unroll
+                    for (int i2 = 1; i2 < K; ++i2)
+#pragma unroll
+                        for (int j2 = i2; j2 > 0; --j2) {
+                            const int lo = min(so[j2 - 1], so[j2]), hi = max(so[j2 - 1], so[j2]);
+                            so[j2 - 1] = lo;
+                            so[j2] = hi;
+                        }
+#pragma unroll
+                    for (int q1 = 0; q1 < K - 1; ++q1) {
+                        const int row = s_rowoff[so[q1]];
+#pragma unroll
+                        for (int q2 = q1 + 1; q2 < K; ++q2) {
+                            const int wi = row + so[q2];
+                            if (a.packed) atomicAdd(&s_tri[wi >> 1], 1u << (16 * (wi & 1)));
+                            else atomicAdd(&tri[wi], 1u);
+                        }
+                    }
+                }
                 emit_words<kRE, K, true>(sel, valid, lane, a.bits + (int64_t)layer * kRE * a.W + w, a.W,
                                          cnt);
             }
@@ -265,9 +296,19 @@ router_sig_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constan
         for (int r = 0; r < kRE / 32; ++r)
             if (cnt[r]) {
                 const int e = 32 * r + lane;
-                atomicAdd(&tri[s_rowoff[e] + e], cnt[r]);
+                const int wi = s_rowoff[e] + e;
+                if (a.packed) atomicAdd(&s_tri[wi >> 1], cnt[r] << (16 * (wi & 1)));
+                else atomicAdd(&tri[wi], cnt[r]);
                 atomicAdd(&a.counts[layer * kRE + e], (int)cnt[r]);
             }
+        if (a.packed) {
+            // all epilogue warps have counted: the triangle out, unpacked
+            asm volatile("bar.sync 1, %0;" ::"n"(kREpiWarps * 32) : "memory");
+            for (int q = threadIdx.x - 64; q < RC::kCoocWords / 2; q += kREpiWarps * 32) {
+                const uint32_t v = s_tri[q];
+                reinterpret_cast<uint2 *>(tri)[q] = make_uint2(v & 0xFFFFu, v >> 16);
+            }
+        }
     }
     tc_fence_before();
     __syncthreads();
@@ -335,13 +376,18 @@ cudaError_t launch_router_signatures(const void *X, const void *Wr, int H, float
     a.T = p.T;
     a.W = p.W;
     a.H = H;
+    const int ctas = router_ctas_per_problem(p);
+    // 16-bit shared counters hold a CTA's counts while its range is below
+    // 65536 tokens; DOLOSS_ROUTER_COOC=global selects the L2 reductions
+    const char *mode = std::getenv("DOLOSS_ROUTER_COOC");
+    const bool force_global = mode && std::strcmp(mode, "global") == 0;
+    a.packed = !force_global && 32 * ((p.W + ctas - 1) / ctas) <= 65535;
     a.bits = bits;
     a.idx = idx;
     a.cooc = cooc;
     a.counts = counts;
     a.zero = zero;
     a.status = status;
-    const int ctas = router_ctas_per_problem(p);
     switch (p.k) {
         case 1: return run_router<1>(xm, wm, zm, a, ctas, p.L, s);
         case 2: return run_router<2>(xm, wm, zm, a, ctas, p.L, s);

@@ -143,3 +143,18 @@ def test_router_backward_full_size(dl):
     check_router_grads(dW[0], dX[0], X[0], W[0], out.dlogits[0],
                        cols=np.sort(rng.choice(H, 48, replace=False)),
                        rows=np.sort(rng.choice(T, 256, replace=False)))
+
+
+def test_router_cooc_paths_agree(dl, monkeypatch):
+    """The co-occurrence counts in 16-bit shared counters (the default for CTA
+    ranges below 65536 tokens) and as L2 reductions (DOLOSS_ROUTER_COOC=global,
+    the path of longer ranges) give the same D, counts and loss."""
+    X, W = workloads.router_inputs(20000, 256, 128, 2, seed=11, device="cuda")
+    z1, a = dl.router_forward_backward(X, W, 8)
+    assert dl.device_status(a.workspace) == 0
+    monkeypatch.setenv("DOLOSS_ROUTER_COOC", "global")
+    z2, b = dl.router_forward_backward(X, W, 8)
+    assert dl.device_status(b.workspace) == 0
+    assert torch.equal(z1, z2)
+    for name in ("bits", "counts", "D", "loss", "origin_do", "dlogits"):
+        assert torch.equal(getattr(a, name), getattr(b, name)), name
