@@ -89,6 +89,15 @@ do_status do_signatures(const float *logits, int64_t T, int32_t E, int32_t k, in
 do_status do_pairwise_hamming(const uint32_t *bits, int64_t T, int32_t E, int32_t L,
                               int32_t *D, void *stream);
 
+/* D += the Hamming matrix of bits (exact integer adds).  Sums the distance
+ * matrices of several token windows, e.g. the micro-batches of one gradient
+ * accumulation window (App. batch ablation: the effective batch of G is
+ * micro-batch x ranks x accumulation steps); G is additive over disjoint
+ * token windows.  D must hold the running sum (zero before the first
+ * window); the caller keeps every row sum within int32. */
+do_status do_pairwise_hamming_accumulate(const uint32_t *bits, int64_t T, int32_t E, int32_t L,
+                                         int32_t *D, void *stream);
+
 /* Step 3 (Sec. 3.1.3, Eq. do_loss; Sec. 3.1.4, Eq. global_do):
  *   L_DO = 1/(T^2 k) sum_i sum_j G_ij C_ij,  C_ij = sum_t p_it (f_it - f_jt),
  * with G = d_scale * D held constant (detached) and p the dense router

@@ -146,6 +146,17 @@ do_status do_pairwise_hamming(const uint32_t *bits, int64_t T, int32_t E, int32_
     return from_cuda(dol::launch_hamming(bits, p, D, (cudaStream_t)stream));
 }
 
+do_status do_pairwise_hamming_accumulate(const uint32_t *bits, int64_t T, int32_t E, int32_t L,
+                                         int32_t *D, void *stream) {
+    NvtxRange nvtx("do_pairwise_hamming_accumulate");
+    Problem p;
+    do_status st = check_sizes(T, E, 1, L, &p);
+    if (st != DO_OK) return st;
+    if (!bits || !D) return DO_ERR_INVALID_ARG;
+    if (!aligned(bits, 4) || !aligned(D, 4)) return DO_ERR_INVALID_ARG;
+    return from_cuda(dol::launch_hamming_accumulate(bits, p, D, nullptr, (cudaStream_t)stream));
+}
+
 do_status do_loss_fwd_bwd(const float *logits, const uint32_t *bits, const int32_t *D, int64_t T,
                           int32_t E, int32_t k, int32_t L, int32_t gate, float d_scale,
                           float grad_scale, float *loss, int64_t *origin_do, float *dlogits,

@@ -25,6 +25,7 @@ EXPORTS = {
     # name: (argtypes, restype)
     "do_signatures": (["p", "i64", "i32", "i32", "i32", "p", "p", "p"], "i32"),
     "do_pairwise_hamming": (["p", "i64", "i32", "i32", "p", "p"], "i32"),
+    "do_pairwise_hamming_accumulate": (["p", "i64", "i32", "i32", "p", "p"], "i32"),
     "do_loss_fwd_bwd": (["p", "p", "p", "i64", "i32", "i32", "i32", "i32", "f32", "f32", "p",
                          "p", "p", "p", "sz", "p"], "i32"),
     "do_forward_backward": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p", "p", "p",
@@ -476,3 +477,35 @@ def global_forward_backward(logits, k, gate=GATE_SIGMOID_NORM, grad_scale=1.0, g
     loss, _, dz = loss_fwd_bwd(z, bits, D, k, gate, d_scale=d_scale, grad_scale=grad_scale,
                                with_origin=False)
     return loss, dz, D, counts
+
+
+def window_forward_backward(logits_list, k, gate=GATE_SIGMOID_NORM, grad_scale=1.0, group=None):
+    """Global-DO over a gradient-accumulation window (Sec. 3.1.4, Eq. global_do;
+    App. batch ablation): the Hamming matrices of the window's micro-batches
+    are summed (do_pairwise_hamming_accumulate), then summed over the ranks of
+    `group`, and every micro-batch's loss and gradient use that matrix with
+    d_scale = 1 / (ranks x micro-batches) and m = its own token count.
+    logits_list: the window's micro-batches, each [L,T,E] or [T,E] on the GPU.
+    Returns (losses: list of [L] fp32, dlogits: list of [L,T,E], D [L,E,E])."""
+    zs = [_as3d(z) for z in logits_list]
+    if not zs:
+        raise ValueError("an empty window")
+    L, _, E = zs[0].shape
+    D = torch.zeros(L, E, E, dtype=torch.int32, device=zs[0].device)
+    sigs = []
+    for z in zs:
+        if z.shape[0] != L or z.shape[2] != E:
+            raise ValueError("the window's micro-batches must share L and E")
+        bits, _ = signatures(z, k)
+        _check("do_pairwise_hamming_accumulate", lib().do_pairwise_hamming_accumulate(
+            bits.data_ptr(), z.shape[1], E, L, D.data_ptr(), _stream(z)))
+        sigs.append(bits)
+    D, d_rank = all_reduce_distances(D, group)
+    d_scale = d_rank / len(zs)
+    losses, grads = [], []
+    for z, bits in zip(zs, sigs):
+        loss, _, dz = loss_fwd_bwd(z, bits, D, k, gate, d_scale=d_scale, grad_scale=grad_scale,
+                                   with_origin=False)
+        losses.append(loss)
+        grads.append(dz)
+    return losses, grads, D

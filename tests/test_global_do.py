@@ -87,3 +87,27 @@ def test_single_rank_global_do_equals_local_path():
     assert float(loss[0]) == pytest.approx(float(ref.loss[0]), rel=1e-5)
     err = (dz - ref.dlogits).abs().max() / ref.dlogits.abs().max()
     assert float(err) <= 1e-5
+
+
+@pytest.mark.gpu
+def test_accumulation_window_matches_oracle():
+    """A window of three micro-batches (ragged sizes): D is the sum of their
+    Hamming matrices, and each micro-batch's loss and gradient are Eq. global_do
+    with that matrix, d_scale = 1/3 and m its own token count."""
+    import oracle
+    import paper_2609_32398_gb300.doloss as dl
+    from paper_2609_32398_gb300 import workloads
+
+    k, E = 8, 128
+    zs = [workloads.random_logits(T, E, seed=T) for T in (4096, 1000 + 33, 2048)]
+    losses, grads, D = dl.window_forward_backward([z.cuda() for z in zs], k)
+    D_ref = sum(oracle.hamming(oracle.select(z[0].numpy(), k)) for z in zs)
+    assert np.array_equal(D[0].cpu().numpy(), D_ref)
+    for z, loss, dz in zip(zs, losses, grads):
+        zl = z[0].numpy()
+        f = oracle.select(zl, k)
+        T = zl.shape[0]
+        want = oracle.loss(D_ref, oracle.direction(zl, f), T, k, d_scale=1.0 / 3)
+        assert abs(float(loss[0]) - want) <= 1e-5 * abs(want)
+        g = oracle.gate_backward(zl, oracle.dloss_dp(D_ref, f, T, k, d_scale=1.0 / 3))
+        assert np.abs(dz[0].double().cpu().numpy() - g).max() <= 1e-4 * np.abs(g).max()
