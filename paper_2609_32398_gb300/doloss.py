@@ -509,3 +509,31 @@ def window_forward_backward(logits_list, k, gate=GATE_SIGMOID_NORM, grad_scale=1
         losses.append(loss)
         grads.append(dz)
     return losses, grads, D
+
+
+class _DOLossFunction(torch.autograd.Function):
+    """The DO-loss of one call as an autograd node: the forward runs steps 1-3
+    (the gradient with grad_scale = 1 comes out of the same pass), and the
+    backward returns it times the incoming gradient of each problem's loss."""
+
+    @staticmethod
+    def forward(ctx, logits, k, gate):
+        squeeze = logits.dim() == 2
+        out = forward_backward(logits.detach(), k, gate, 1.0)
+        ctx.save_for_backward(out.dlogits)
+        ctx.squeeze = squeeze
+        return out.loss[0].clone() if squeeze else out.loss.clone()
+
+    @staticmethod
+    def backward(ctx, grad):
+        (dz,) = ctx.saved_tensors
+        dz = dz * grad.reshape(-1, 1, 1).to(dz.dtype)
+        return (dz[0] if ctx.squeeze else dz), None, None
+
+
+def do_loss(logits: torch.Tensor, k: int, gate=GATE_SIGMOID_NORM) -> torch.Tensor:
+    """The DO-loss (Sec. 3.1.3, Eq. do_loss) of router logits [T,E] or [L,T,E]
+    (fp32, CUDA) as a differentiable tensor: a scalar, or [L] per problem.
+    Multiply by the loss weight and add to the training objective; the
+    gradient reaches the logits through autograd."""
+    return _DOLossFunction.apply(_as3d(logits) if logits.dim() == 3 else logits, k, gate)

@@ -301,3 +301,22 @@ def test_async_host_entry_matches_the_synchronous_one(dl, T, E, k, gate):
         loss, flags = dl.host_result(r, 1)
         assert flags == 0
         assert torch.equal(loss, want)
+
+
+def test_autograd_wrapper_gives_the_path_gradient(dl):
+    """do_loss as an autograd node: the loss of do_forward_backward, and the
+    gradient times the incoming gradient (here the loss weight 0.3, and one
+    weight per layer for a batched call)."""
+    z = workloads.random_logits(4096 + 33, 128, L=2, seed=21).cuda()
+    ref = dl.forward_backward(z, 8, 0)
+    x = z.clone().requires_grad_(True)
+    loss = dl.do_loss(x, 8)
+    assert torch.equal(loss, ref.loss)
+    (loss * torch.tensor([0.3, 2.0], device="cuda")).sum().backward()
+    assert torch.allclose(x.grad[0], 0.3 * ref.dlogits[0], rtol=1e-6, atol=0)
+    assert torch.allclose(x.grad[1], 2.0 * ref.dlogits[1], rtol=1e-6, atol=0)
+    y = z[0].clone().requires_grad_(True)
+    l1 = dl.do_loss(y, 8)
+    assert l1.dim() == 0 and float(l1.detach()) == float(ref.loss[0])
+    (0.3 * l1).backward()
+    assert torch.allclose(y.grad, 0.3 * ref.dlogits[0], rtol=1e-6, atol=0)
