@@ -67,6 +67,7 @@ def _load():
             "oracle_route": ([P, I64, I32, I32, I32, P, P], None),
             "oracle_dispatch": ([P, I64, I32, I32, P, P, P], None),
             "oracle_bf16_to_double": ([P, I64, P], None),
+            "oracle_direction_mode": ([P, P, I64, I64, I32, I32, I32, P], None),
             "oracle_router_logits": ([P, P, I64, I32, I32, P], None),
             "oracle_router_grad": ([P, P, P, I64, I32, I32, P, P], None),
         }
@@ -256,3 +257,14 @@ def router_grad(X, Wr, dz, with_dx=False):
     _load().oracle_router_grad(px, pw, pd, T, H, E, dW.ctypes.data,
                                dX.ctypes.data if dX is not None else None)
     return (dW, dX) if with_dx else dW
+
+
+def direction_mode(z, f, gate_kind=GATE_SIGMOID_NORM, mode=0):
+    """C_ij with the dense p (mode 0, the path's reading) or the re-normalized
+    top-K weights (mode 1)."""
+    z, pz = _c(z, np.float32)
+    f, pf = _c(f, np.uint8)
+    T, E = z.shape
+    C = np.zeros((E, E), np.float64)
+    _load().oracle_direction_mode(pz, pf, 0, T, E, gate_kind, mode, C.ctypes.data)
+    return C

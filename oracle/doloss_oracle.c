@@ -359,3 +359,28 @@ void oracle_router_grad(const uint16_t *X, const uint16_t *Wr, const double *dz,
             dX[t * H + h] = acc;
         }
 }
+
+/* The other reading of which p enters C_ij (Sec. 3.1.1 describes both the
+ * dense normalized p and, after Top-K, the K chosen values re-normalized):
+ * mode 0 takes the dense p of gate_row, mode 1 the re-normalized top-K
+ * weights (zero for the experts not chosen).  C is [E][E], accumulated over
+ * tokens [t0, t1).  The path implements mode 0; mode 1 is kept so that the
+ * reading can be checked against App. C.2 (idle experts receive gradient). */
+void oracle_direction_mode(const float *z, const uint8_t *f, int64_t t0, int64_t t1, int32_t E,
+                           int32_t gate, int32_t mode, double *C)
+{
+    double *p = (double *)malloc(sizeof(double) * (size_t)E);
+    for (int64_t t = t0; t < t1; ++t) {
+        const uint8_t *ft = f + t * E;
+        gate_row(z + t * E, E, gate, p);
+        if (mode == 1) {
+            double kept = 0.0;
+            for (int32_t i = 0; i < E; ++i) kept += ft[i] ? p[i] : 0.0;
+            for (int32_t i = 0; i < E; ++i) p[i] = ft[i] ? p[i] / kept : 0.0;
+        }
+        for (int32_t i = 0; i < E; ++i)
+            for (int32_t j = 0; j < E; ++j)
+                C[(int64_t)i * E + j] += p[i] * ((double)ft[i] - (double)ft[j]);
+    }
+    free(p);
+}

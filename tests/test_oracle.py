@@ -339,3 +339,40 @@ def test_global_do_scaling_is_linear_in_the_summed_matrix():
     C = oracle.direction(z, f)
     both = oracle.loss(D1 + D2, C, T, k, d_scale=0.5)
     assert both == pytest.approx(0.5 * (oracle.loss(D1, C, T, k) + oracle.loss(D2, C, T, k)), rel=1e-13)
+
+
+def test_dense_p_reading_against_the_renormalized_one():
+    """Sec. 3.1.1 gives p both dense and, after Top-K, re-normalized over the K
+    chosen experts.  Mode 0 (dense) is the path's reading; checked here: it
+    equals oracle.direction, and only it gives the idle experts of App. C.2 a
+    gradient.  With re-normalized weights the experts outside a token's Top-K
+    have p = 0 whatever their logits, and every idle expert's logit gradient
+    (through the surrogate, G detached) vanishes; with the dense p it is
+    negative (App. C.2: idle experts are pulled up)."""
+    T, E, k = 60, 8, 2
+    z = rand_z(T, E, 31)
+    z[:, 6:] -= 6.0                                  # experts 6 and 7 never chosen
+    f = oracle.select(z, k)
+    assert not f[:, 6:].any()
+    D = oracle.hamming(f)
+    C0 = oracle.direction_mode(z, f, mode=0)
+    np.testing.assert_allclose(C0, oracle.direction(z, f), rtol=1e-14, atol=1e-14)
+
+    def loss_of(zz, mode):
+        return oracle.loss(D, oracle.direction_mode(zz.astype(np.float32), f, mode=mode), T, k)
+
+    for mode, sign in ((0, -1), (1, 0)):
+        for i in (6, 7):
+            h = 1e-2
+            zp, zm = z.astype(np.float64).copy(), z.astype(np.float64).copy()
+            zp[:, i] += h
+            zm[:, i] -= h
+            g = (loss_of(zp, mode) - loss_of(zm, mode)) / (2 * h)
+            if sign == 0:
+                assert abs(g) < 1e-12                # rounding of the cancelled normaliser only
+            else:
+                assert g < -1e-6
+    # with re-normalized weights the chosen mass is one for every token
+    # (App. A: s_K = 1), so sum C = m (n - k) exactly
+    C1 = oracle.direction_mode(z, f, mode=1)
+    assert C1.sum() == pytest.approx(T * (E - k), rel=1e-12)
