@@ -537,3 +537,15 @@ def do_loss(logits: torch.Tensor, k: int, gate=GATE_SIGMOID_NORM) -> torch.Tenso
     Multiply by the loss weight and add to the training objective; the
     gradient reaches the logits through autograd."""
     return _DOLossFunction.apply(_as3d(logits) if logits.dim() == 3 else logits, k, gate)
+
+
+def offdiag_variance(origin_do, T: int, E: int, k: int):
+    """Variance of the off-diagonal entries of a local Hamming matrix, from
+    Eq. origin_do (the exact sum of their squares) and Eq. zero_sum (their sum
+    is 2 T k (E - k)): Var = origin_do / (E (E - 1)) - mean^2.  origin_do may
+    be an int, or an int64 tensor [L] (returned as float64 [L])."""
+    n = E * (E - 1)
+    mean = 2.0 * T * k * (E - k) / n
+    if isinstance(origin_do, torch.Tensor):
+        return origin_do.double() / n - mean * mean
+    return int(origin_do) / n - mean * mean

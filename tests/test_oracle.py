@@ -376,3 +376,15 @@ def test_dense_p_reading_against_the_renormalized_one():
     # (App. A: s_K = 1), so sum C = m (n - k) exactly
     C1 = oracle.direction_mode(z, f, mode=1)
     assert C1.sum() == pytest.approx(T * (E - k), rel=1e-12)
+
+
+def test_offdiag_variance_from_origin_do():
+    """Eq. origin_do with Eq. zero_sum gives the variance of the off-diagonal
+    distances without reading D (numpy's variance of the entries pins it)."""
+    from paper_2609_32398_gb300.doloss import offdiag_variance
+
+    for T, E, k in ((97, 8, 2), (500, 33, 5)):
+        f = oracle.select(rand_z(T, E, T + E), k)
+        D = oracle.hamming(f)
+        off = D[~np.eye(E, dtype=bool)].astype(np.float64)
+        assert offdiag_variance(oracle.origin_do(D), T, E, k) == pytest.approx(off.var(), rel=1e-12)
