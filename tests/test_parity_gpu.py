@@ -320,3 +320,24 @@ def test_autograd_wrapper_gives_the_path_gradient(dl):
     assert l1.dim() == 0 and float(l1.detach()) == float(ref.loss[0])
     (0.3 * l1).backward()
     assert torch.allclose(y.grad, 0.3 * ref.dlogits[0], rtol=1e-6, atol=0)
+
+
+def test_first_size_past_the_tensor_core_limit(dl):
+    """T = 66053 at E = 128: (E - 1) T reaches 2^23, where the two-piece fp16
+    split of D' stops being exact, so the fused path takes the ALU gradient
+    pass; it must still match the oracle."""
+    T, E, k = 66053, 128, 8
+    z = workloads.random_logits(T, E, seed=66053)
+    out = gpu_run(dl, z, k, 0)
+    assert_layer(out, 0, z[0].numpy(), k, 0)
+
+
+@pytest.mark.parametrize("T,E,k", [(32, 32, 2), (1, 8, 2)])
+def test_largest_batch_of_problems(dl, T, E, k):
+    """L = 65535 problems in one call (the grid's y/z limit): the fast kernels
+    (E = 32) and the generic ones (E = 8), sampled layers against the oracle."""
+    L = 65535
+    z = workloads.random_logits(T, E, L=L, seed=L + E)
+    out = gpu_run(dl, z, k, 0)
+    for l in np.random.default_rng(E).choice(L, 40, replace=False).tolist() + [0, L - 1]:
+        assert_layer(out, l, z[l].numpy(), k, 0)
