@@ -7,8 +7,8 @@
 // signatures kernel.  A CTA owns 32 consecutive triangle words; its 32 warps
 // each sum a strided subset of the partials with independent loads, and the
 // 32 warp sums are added in a fixed order, so D is an exact integer result
-// independent of scheduling.  The kernel writes both halves of the symmetric
-// D and the counts.
+// independent of scheduling (every load of a warp is issued before any add).
+// The kernel writes both halves of the symmetric D and the counts.
 #include <cuda_fp16.h>
 
 #include "dol_internal.cuh"
@@ -19,6 +19,7 @@ namespace {
 
 constexpr int kRedWarps = 32;
 constexpr int kRedThreads = kRedWarps * 32;
+static_assert(kMaxSigCtas <= 8 * kRedWarps, "a warp adds at most eight partials");
 
 __device__ __forceinline__ void put_pieces(unsigned char *img, int n, int k, bool diag, int v) {
     int h, l;
@@ -41,18 +42,18 @@ cooc_reduce_kernel(const uint32_t *__restrict__ partials, int P1, const int *__r
     pdl_wait();
     pdl_trigger();
     if ((int)threadIdx.x < E) s_n[threadIdx.x] = n_acc[(size_t)layer * E + threadIdx.x];
-    uint32_t acc[4] = {0u, 0u, 0u, 0u};
-    if (word < kWords) {
-        const uint32_t *base = partials + (size_t)layer * P1 * kWords + word;
-        for (int p0 = wp; p0 < P1; p0 += 4 * kRedWarps) {
+    // every partial this warp adds (P1 <= 8 x 32) is requested at once
+    uint32_t v[8];
+    const uint32_t *base = partials + (size_t)layer * P1 * kWords + word;
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int p = p0 + u * kRedWarps;
-                if (p < P1) acc[u] += __ldg(base + (size_t)p * kWords);
-            }
-        }
+    for (int u = 0; u < 8; ++u) {
+        const int p = wp + u * kRedWarps;
+        v[u] = (word < kWords && p < P1) ? __ldg(base + (size_t)p * kWords) : 0u;
     }
-    s_sum[wp][e] = acc[0] + acc[1] + acc[2] + acc[3];
+    uint32_t acc = 0u;
+#pragma unroll
+    for (int u = 0; u < 8; ++u) acc += v[u];
+    s_sum[wp][e] = acc;
     __syncthreads();
     if (wp != 0) return;
     long long sq = 0;  // this word's part of sum_{a != b} D_ab^2
