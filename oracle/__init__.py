@@ -68,6 +68,7 @@ def _load():
             "oracle_dispatch": ([P, I64, I32, I32, P, P, P], None),
             "oracle_bf16_to_double": ([P, I64, P], None),
             "oracle_direction_mode": ([P, P, I64, I64, I32, I32, I32, P], None),
+            "oracle_route_backward": ([P, P, P, I64, I32, I32, I32, P], None),
             "oracle_router_logits": ([P, P, I64, I32, I32, P], None),
             "oracle_router_grad": ([P, P, P, I64, I32, I32, P, P], None),
         }
@@ -268,3 +269,16 @@ def direction_mode(z, f, gate_kind=GATE_SIGMOID_NORM, mode=0):
     C = np.zeros((E, E), np.float64)
     _load().oracle_direction_mode(pz, pf, 0, T, E, gate_kind, mode, C.ctypes.data)
     return C
+
+
+def route_backward(z, ids, g, gate_kind=GATE_SIGMOID_NORM):
+    """dz [T,E] float64: the gradient of the combine weights to the logits for
+    the upstream gradient g [T,k] of the weights."""
+    z, pz = _c(z, np.float32)
+    ids, pi = _c(ids, np.int32)
+    g, pg = _c(g, np.float64)
+    T, E = z.shape
+    k = ids.shape[1]
+    dz = np.empty((T, E), np.float64)
+    _load().oracle_route_backward(pz, pi, pg, T, E, k, gate_kind, dz.ctypes.data)
+    return dz

@@ -384,3 +384,48 @@ void oracle_direction_mode(const float *z, const uint8_t *f, int64_t t0, int64_t
     }
     free(p);
 }
+
+/* Gradient of the combine weights (Sec. 3.1.1: w_tq = p_{e_q,t} / sum_q' p_{e_q',t})
+ * to the logits, for an upstream gradient g [T][k] of the weights: with the
+ * dense p written out, dz_tl = sum_q g_tq d w_tq / d z_tl for every expert l
+ * (the experts not chosen have a zero derivative, the dense normaliser
+ * cancelling), computed entry by entry in double:
+ *   sigmoid-norm: w_q = s_q / S,  S = sum of the chosen s,
+ *                 d w_q / d z_l = [l chosen] s_l (1 - s_l) (delta_ql - w_q) / S
+ *   softmax:      w_q = exp(z_q) / sum of the chosen exp(z),
+ *                 d w_q / d z_l = [l chosen] w_q (delta_ql - w_l)
+ * ids [T][k] are the chosen experts; dz is [T][E]. */
+void oracle_route_backward(const float *z, const int32_t *ids, const double *g, int64_t T,
+                           int32_t E, int32_t k, int32_t gate, double *dz)
+{
+    double *w = (double *)malloc(sizeof(double) * (size_t)k);
+    double *sv = (double *)malloc(sizeof(double) * (size_t)k);
+    for (int64_t t = 0; t < T; ++t) {
+        const float *zt = z + t * (int64_t)E;
+        const int32_t *it = ids + t * (int64_t)k;
+        const double *gt = g + t * (int64_t)k;
+        double *dt = dz + t * (int64_t)E;
+        for (int32_t l = 0; l < E; ++l) dt[l] = 0.0;
+        double S = 0.0, zmax = (double)zt[it[0]];
+        for (int32_t q = 0; q < k; ++q)
+            if ((double)zt[it[q]] > zmax) zmax = (double)zt[it[q]];
+        for (int32_t q = 0; q < k; ++q) {
+            double v = (double)zt[it[q]];
+            sv[q] = gate == GATE_SOFTMAX ? exp(v - zmax) : 1.0 / (1.0 + exp(-v));
+            S += sv[q];
+        }
+        for (int32_t q = 0; q < k; ++q) w[q] = sv[q] / S;
+        for (int32_t m = 0; m < k; ++m) {     /* l = ids[m], a chosen expert */
+            double acc = 0.0;
+            for (int32_t q = 0; q < k; ++q) {
+                double delta = (q == m) ? 1.0 : 0.0;
+                double J = gate == GATE_SOFTMAX ? w[q] * (delta - w[m])
+                                                : sv[m] * (1.0 - sv[m]) * (delta - w[q]) / S;
+                acc += gt[q] * J;
+            }
+            dt[it[m]] = acc;
+        }
+    }
+    free(w);
+    free(sv);
+}

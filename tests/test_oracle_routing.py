@@ -108,3 +108,30 @@ def test_dispatch_is_a_stable_sort_by_expert(T, E, k):
         seg = rows[offsets[e]:offsets[e + 1]]
         assert (np.diff(seg) > 0).all()             # each token once, ascending
         assert all(e in ids[t] for t in seg)
+
+
+@pytest.mark.parametrize("gate", [oracle.GATE_SIGMOID_NORM, oracle.GATE_SOFTMAX])
+@pytest.mark.parametrize("E,k", [(8, 2), (33, 5), (128, 8)])
+def test_route_backward_matches_autograd(gate, E, k):
+    """The combine weights' gradient to the logits against torch float64
+    autograd through the paper's definition (dense p, then re-normalized over
+    the chosen experts), the selection held fixed."""
+    T = 50
+    z = rand_z(T, E, seed=E * 3 + k + gate)
+    ids, _ = oracle.route(z, k, gate)
+    g = np.random.default_rng(E + k).standard_normal((T, k))
+    zt = torch.from_numpy(z.astype(np.float64)).requires_grad_(True)
+    if gate == oracle.GATE_SOFTMAX:
+        p = torch.softmax(zt, dim=1)
+    else:
+        s = torch.sigmoid(zt)
+        p = s / s.sum(1, keepdim=True)
+    pc = torch.gather(p, 1, torch.from_numpy(ids.astype(np.int64)))
+    w = pc / pc.sum(1, keepdim=True)
+    (w * torch.from_numpy(g)).sum().backward()
+    dz = oracle.route_backward(z, ids, g, gate)
+    np.testing.assert_allclose(dz, zt.grad.numpy(), rtol=1e-10, atol=1e-13)
+    # the experts not chosen get nothing
+    mask = np.ones_like(dz, dtype=bool)
+    np.put_along_axis(mask, ids.astype(np.int64), False, axis=1)
+    assert (dz[mask] == 0.0).all()
