@@ -391,7 +391,8 @@ void oracle_direction_mode(const float *z, const uint8_t *f, int64_t t0, int64_t
  * (the experts not chosen have a zero derivative, the dense normaliser
  * cancelling), computed entry by entry in double:
  *   sigmoid-norm: w_q = s_q / S,  S = sum of the chosen s,
- *                 d w_q / d z_l = [l chosen] s_l (1 - s_l) (delta_ql - w_q) / S
+ *                 d w_q / d z_l = [l chosen] s_l (1 - s_l) (delta_ql - w_q) / S,
+ *                 with 1 - s_l evaluated as sigmoid(-z_l)
  *   softmax:      w_q = exp(z_q) / sum of the chosen exp(z),
  *                 d w_q / d z_l = [l chosen] w_q (delta_ql - w_l)
  * ids [T][k] are the chosen experts; dz is [T][E]. */
@@ -419,8 +420,10 @@ void oracle_route_backward(const float *z, const int32_t *ids, const double *g, 
             double acc = 0.0;
             for (int32_t q = 0; q < k; ++q) {
                 double delta = (q == m) ? 1.0 : 0.0;
-                double J = gate == GATE_SOFTMAX ? w[q] * (delta - w[m])
-                                                : sv[m] * (1.0 - sv[m]) * (delta - w[q]) / S;
+                /* 1 - sigmoid(v) written as sigmoid(-v): no cancellation for large v */
+                double J = gate == GATE_SOFTMAX
+                               ? w[q] * (delta - w[m])
+                               : sv[m] * (1.0 / (1.0 + exp((double)zt[it[m]]))) * (delta - w[q]) / S;
                 acc += gt[q] * J;
             }
             dt[it[m]] = acc;

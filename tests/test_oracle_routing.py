@@ -135,3 +135,22 @@ def test_route_backward_matches_autograd(gate, E, k):
     mask = np.ones_like(dz, dtype=bool)
     np.put_along_axis(mask, ids.astype(np.int64), False, axis=1)
     assert (dz[mask] == 0.0).all()
+
+
+@pytest.mark.parametrize("c", [0.0, 3.0, 60.0, -60.0])
+@pytest.mark.parametrize("gate", [oracle.GATE_SIGMOID_NORM, oracle.GATE_SOFTMAX])
+def test_route_backward_equal_chosen_logits_closed_form(c, gate):
+    """All chosen logits equal to c (the rest far below): w = 1/k, so
+    dz_l = (1/k) (g_l - mean g) for softmax and (1/k) sigmoid(-c) (g_l - mean g)
+    for sigmoid-norm, at every size of c (1 - sigmoid(c) is tiny for c = 60)."""
+    T, E, k = 20, 16, 5
+    z = np.full((T, E), c - 200.0, np.float32)
+    z[:, 3:3 + k] = c
+    ids, _ = oracle.route(z, k, gate)
+    assert (np.sort(ids, 1) == np.arange(3, 3 + k)).all()
+    g = np.random.default_rng(1).standard_normal((T, k))
+    dz = oracle.route_backward(z, ids, g, gate)
+    factor = 1.0 if gate == oracle.GATE_SOFTMAX else 1.0 / (1.0 + np.exp(c))
+    want = (g - g.mean(1, keepdims=True)) / k * factor
+    np.testing.assert_allclose(np.take_along_axis(dz, ids.astype(np.int64), axis=1), want,
+                               rtol=1e-12, atol=0)
