@@ -63,6 +63,13 @@ def routing_bytes(T, E, k, L=1):
     return L * (4 * T * E + 16 * T * k + 8 * E + 4)
 
 
+def route_backward_bytes(T, E, k, L=1, accumulate=False):
+    """Bytes of the combine weights' backward: expert ids, their gradient and
+    the k chosen logits read (4Tk each); then either every dlogits entry
+    written (4TE) or the k chosen entries read and written in place (8Tk)."""
+    return L * (12 * T * k + (8 * T * k if accumulate else 4 * T * E))
+
+
 ROUTER_HIDDEN = 2048  # the 30BA3B router's input width (hidden size, Sec. 4.1)
 
 
@@ -89,6 +96,7 @@ UNIT_SOURCES = {
                             "loss.cu", "tma.cuh", "tma_host.cu", "dol_internal.cuh", "api.cu"],
     "do_routing": ["sig_fast.cuh", "route.cu", "signatures.cu", "tma.cuh", "tma_host.cu",
                    "dol_internal.cuh", "api.cu"],
+    "do_route_backward": ["route_bwd.cu", "dol_internal.cuh", "api.cu"],
     "do_router_forward_backward": ["router.cu", "sig_fast.cuh", "cooc_reduce.cu", "loss_mma.cu",
                                    "loss.cu", "tma.cuh", "tma_host.cu", "dol_internal.cuh",
                                    "api.cu"],
@@ -308,6 +316,14 @@ def run_ours(args, rank, world, local):
             def call(i):
                 dl.router_forward_backward(X, Wr, k, w.gate, 1.0, out=sets[0][1], logits=zr)
             ws = sets[0][1].workspace
+        elif args.quick_path == "route_bwd":
+            route = dl.routing(sets[0][0], k, w.gate)
+            gq = torch.randn(L, T, k, device=dev)
+
+            def call(i):
+                dl.route_backward(sets[i % N_SETS][0], route.expert_ids, gq, w.gate,
+                                  dlogits=sets[i % N_SETS][1].dlogits)
+            ws = route.workspace
         else:
             route = dl.Routing(L, T, E, k, dev)
             if args.quick_path == "routing":
@@ -405,6 +421,23 @@ def run_ours(args, rank, world, local):
         sets[r % N_SETS][0], k, w.gate, 1.0, out=sets[r % N_SETS][1], route=routes[r % N_SETS]))
     plain_ms = time_calls(lambda r: dl.forward_backward(sets[r % N_SETS][0], k, w.gate, 1.0,
                                                         out=sets[r % N_SETS][1]))
+    # The combine weights' backward to the logits: written over a dlogits
+    # buffer, and added into the DO-loss step's dlogits (the training use).
+    gqs = [torch.randn(L, T, k, device=dev, generator=torch.Generator(dev).manual_seed(r))
+           for r in range(N_SETS)]
+    rb_flags = torch.zeros(1, dtype=torch.int32, device=dev)
+    rbwd_ms = time_calls(lambda r: dl.route_backward(
+        sets[r % N_SETS][0], routes[r % N_SETS].expert_ids, gqs[r % N_SETS], w.gate,
+        dlogits=sets[r % N_SETS][1].dlogits, status_flags=rb_flags))
+    rbwd_acc_ms = time_calls(lambda r: dl.route_backward(
+        sets[r % N_SETS][0], routes[r % N_SETS].expert_ids, gqs[r % N_SETS], w.gate,
+        dlogits=sets[r % N_SETS][1].dlogits, accumulate=True, status_flags=rb_flags))
+    if int(rb_flags[0]) != 0:
+        raise RuntimeError("do_route_backward flagged an expert id out of range")
+    # Context for the fractions at this size: a plain device copy of one
+    # logits-sized buffer into another, in the same rotation of input sets
+    # (the measured peak comes from gigabyte-sized copies).
+    copy_ms = time_calls(lambda r: sets[r % N_SETS][1].dlogits.copy_(sets[r % N_SETS][0]))
     for r in range(N_SETS):
         for ws in (routes[r].workspace, sets[r][1].workspace):
             st = dl.device_status(ws)
@@ -542,6 +575,10 @@ def run_ours(args, rank, world, local):
                          "traffic": profiled_traffic("do_forward_backward")},
             "split_entry_points": {"us": {k_: v * 1e3 for k_, v in stage_ms.items()},
                                    "GB/s": split_gbs},
+            "size_matched_copy": {
+                "what": "torch copy_ of one [L,T,E] fp32 buffer into another, same rotation",
+                "bytes": 8 * T * E * L, "us": copy_ms * 1e3,
+                "GB/s": 8 * T * E * L / (copy_ms * 1e-3) / 1e9},
             "routing": {
                 "entry": "do_routing (selection with ids and combine weights, dispatch order)",
                 "us_per_call": route_ms * 1e3, "tokens_per_s": T * L / (route_ms * 1e-3),
@@ -555,6 +592,20 @@ def run_ours(args, rank, world, local):
                 "fused": {"entry": "do_forward_backward_routed",
                           "us_per_call": routed_ms * 1e3,
                           "us_per_call_without_routing": plain_ms * 1e3},
+                "backward": {
+                    "entry": "do_route_backward (combine weights' gradient to the logits)",
+                    "us_per_call": rbwd_ms * 1e3,
+                    "us_per_call_accumulate": rbwd_acc_ms * 1e3,
+                    "roofline": {"bound": "hbm", "kernel": "route_backward_kernel",
+                                 "achieved": route_backward_bytes(T, E, k, L) / (rbwd_ms * 1e-3) / 1e9,
+                                 "peak": peak, "unit": "GB/s",
+                                 "frac": route_backward_bytes(T, E, k, L) / (rbwd_ms * 1e-3) / 1e9
+                                 / peak,
+                                 "peak_source": peak_src,
+                                 "algorithmic_bytes": route_backward_bytes(T, E, k, L),
+                                 "algorithmic_bytes_accumulate":
+                                     route_backward_bytes(T, E, k, L, accumulate=True),
+                                 "traffic": profiled_traffic("do_route_backward")}},
                 "reps": reps},
             "router_fused": {
                 "entry": "do_router_forward_backward (logits = X W^T on tcgen05 with the signature "
@@ -594,9 +645,11 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--quick", action="store_true",
                     help="run warmup+steps plain steps and exit (for profilers)")
-    ap.add_argument("--quick-path", choices=["loss", "routing", "routed", "router"], default="loss",
+    ap.add_argument("--quick-path", choices=["loss", "routing", "routed", "router", "route_bwd"],
+                    default="loss",
                     help="entry point of --quick: do_forward_backward, do_routing, "
-                         "do_forward_backward_routed or do_router_forward_backward")
+                         "do_forward_backward_routed, do_router_forward_backward or "
+                         "do_route_backward")
     args = ap.parse_args()
     if args.impl == "reference":
         rank = int(os.environ.get("RANK", "0"))

@@ -163,6 +163,33 @@ do_status do_routing(const float *logits, int64_t T, int32_t E, int32_t k, int32
 
 size_t do_routing_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L);
 
+/* Backward of the combine weights of do_routing (Sec. 3.1.1) to the logits,
+ * the selection held fixed.  With g = grad_combine, dot_t = sum_q g_tq w_tq
+ * and l = expert_ids[t][q] a chosen expert:
+ *   sigmoid-norm: dlogits[t][l] = w_tl (1 - sigmoid(z_tl)) (g_tq - dot_t)
+ *   softmax:      dlogits[t][l] = w_tl (g_tq - dot_t)
+ * and 0 for the experts not chosen (the dense normaliser of p cancels).
+ *   logits        [L][T][E] fp32 device, the router logits of the forward pass
+ *   expert_ids    [L][T][k] int32 device, the chosen experts (as do_routing
+ *                 writes them; the ids of a token must be distinct, repeated
+ *                 ids leave the values at those entries unspecified)
+ *   grad_combine  [L][T][k] fp32 device, the gradient of combine
+ *   dlogits       [L][T][E] fp32 device: accumulate = 0 overwrites every
+ *                 entry; accumulate = 1 adds the gradient to the chosen
+ *                 entries only and leaves the rest as they are (so that the
+ *                 call can follow do_forward_backward on the same buffer)
+ * The weights are recomputed in fp32 from the chosen logits (shifted by the
+ * largest one) as do_routing computes them; each result is within a few ulp
+ * of w_tl (|g_tq| + sum_q' |g_tq'| w_tq') times the gate factor.  The result
+ * is identical run to run.  status_flags (device int32, may be NULL): bit 2
+ * (value 4) is ORed in when an expert_ids entry lies outside [0, E) (that
+ * choice is then left out).  4-byte aligned pointers.  Asynchronous on
+ * `stream`. */
+do_status do_route_backward(const float *logits, const int32_t *expert_ids,
+                            const float *grad_combine, int64_t T, int32_t E, int32_t k, int32_t L,
+                            int32_t gate, int32_t accumulate, float *dlogits,
+                            int32_t *status_flags, void *stream);
+
 /* do_forward_backward that also writes the routing outputs of do_routing
  * (expert_ids, combine required; expert_offsets, dispatch_rows, dispatch_pos
  * may each be NULL) from the same selection pass over the logits, so the

@@ -365,6 +365,25 @@ do_status do_routing(const float *logits, int64_t T, int32_t E, int32_t k, int32
     return from_cuda(e);
 }
 
+do_status do_route_backward(const float *logits, const int32_t *expert_ids,
+                            const float *grad_combine, int64_t T, int32_t E, int32_t k, int32_t L,
+                            int32_t gate, int32_t accumulate, float *dlogits,
+                            int32_t *status_flags, void *stream) {
+    NvtxRange nvtx("do_route_backward");
+    Problem p;
+    do_status st = check_sizes(T, E, k, L, &p);
+    if (st != DO_OK) return st;
+    if (gate != DO_GATE_SIGMOID_NORM && gate != DO_GATE_SOFTMAX) return DO_ERR_INVALID_ARG;
+    if (accumulate != 0 && accumulate != 1) return DO_ERR_INVALID_ARG;
+    if (!logits || !expert_ids || !grad_combine || !dlogits) return DO_ERR_INVALID_ARG;
+    if (!aligned(logits, 4) || !aligned(expert_ids, 4) || !aligned(grad_combine, 4) ||
+        !aligned(dlogits, 4) || (status_flags && !aligned(status_flags, 4)))
+        return DO_ERR_INVALID_ARG;
+    return from_cuda(dol::launch_route_backward(logits, expert_ids, grad_combine, p.T * p.L, E, k,
+                                                gate, accumulate, dlogits, status_flags,
+                                                (cudaStream_t)stream));
+}
+
 size_t do_routing_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L) {
     Problem p;
     if (check_sizes(T, E, k, L, &p) != DO_OK) return 0;

@@ -115,6 +115,12 @@ cudaError_t launch_signatures_fast_routed(const float *logits, const Problem &p,
 // programmatic dependents of the previous kernel on `s`.
 int64_t route_chunks(const Problem &p);
 int64_t route_scratch_ints(const Problem &p);
+// Backward of the combine weights to the logits over `rows` token rows
+// (route_bwd.cu); status bit 2 for an id outside [0, E).
+cudaError_t launch_route_backward(const float *z, const int32_t *ids, const float *g, int64_t rows,
+                                  int32_t E, int32_t k, int32_t gate, int32_t accumulate,
+                                  float *dz, int32_t *status_flags, cudaStream_t s);
+
 cudaError_t launch_route_dispatch(const uint32_t *bits, const int *ids, const Problem &p,
                                   int *offsets, int *rows, int *pos, int *scratch,
                                   cudaStream_t s);

@@ -45,6 +45,8 @@ EXPORTS = {
     "do_routing": (["p", "i64", "i32", "i32", "i32", "i32", "p", "p", "p", "p", "p", "p", "p", "sz",
                     "p"], "i32"),
     "do_routing_workspace_size": (["i64", "i32", "i32", "i32"], "sz"),
+    "do_route_backward": (["p", "p", "p", "i64", "i32", "i32", "i32", "i32", "i32", "p", "p", "p"],
+                          "i32"),
     "do_forward_backward_routed": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p", "p",
                                     "p", "p", "p", "p", "p", "p", "p", "p", "p", "sz", "p"], "i32"),
     "do_maxvio": (["p", "p", "i32", "i32", "i32", "p", "p", "p", "p"], "i32"),
@@ -243,6 +245,36 @@ def routing(logits, k, gate=GATE_SIGMOID_NORM, out: Routing | None = None):
         out.counts.data_ptr(), _ptr(out.offsets), _ptr(out.rows), _ptr(out.pos),
         out.workspace.data_ptr(), out.workspace.numel(), _stream(z)))
     return out
+
+
+def route_backward(logits, expert_ids, grad_combine, gate=GATE_SIGMOID_NORM,
+                   dlogits: torch.Tensor | None = None, accumulate=False,
+                   status_flags: torch.Tensor | None = None):
+    """do_route_backward: the gradient of the combine weights (grad_combine
+    [L,T,k] or [T,k] fp32) to the logits [L,T,E], the selection expert_ids
+    held fixed.  With accumulate, it is added to the chosen entries of the
+    given dlogits; otherwise dlogits (made when None) is overwritten.  Returns
+    dlogits."""
+    z = _as3d(logits)
+    L, T, E = z.shape
+    ids = expert_ids.reshape(L, T, -1)
+    g = grad_combine.reshape(L, T, -1)
+    k = ids.shape[2]
+    if ids.dtype != torch.int32 or g.dtype != torch.float32 or g.shape[2] != k:
+        raise ValueError("expert_ids must be int32 and grad_combine float32 of the same [L,T,k]")
+    if not (ids.is_cuda and g.is_cuda and ids.is_contiguous() and g.is_contiguous()):
+        raise ValueError("expert_ids and grad_combine must be contiguous CUDA tensors")
+    if dlogits is None:
+        if accumulate:
+            raise ValueError("accumulate needs the dlogits to add to")
+        dlogits = torch.empty_like(z)
+    if (dlogits.numel() != z.numel() or dlogits.dtype != torch.float32
+            or not dlogits.is_contiguous() or dlogits.device != z.device):
+        raise ValueError("dlogits must be a contiguous float32 tensor shaped like the logits")
+    _check("do_route_backward", lib().do_route_backward(
+        z.data_ptr(), ids.data_ptr(), g.data_ptr(), T, E, k, L, gate, int(bool(accumulate)),
+        dlogits.data_ptr(), _ptr(status_flags), _stream(z)))
+    return dlogits
 
 
 def forward_backward_routed(logits, k, gate=GATE_SIGMOID_NORM, grad_scale=1.0,

@@ -149,3 +149,20 @@ def test_async_host_entry_validates_on_the_host(dl):
                                               None) == INV
     assert lib.do_forward_backward_host_async(fake, 64, 8, 2, 1, 0, 1.0, fake, fake, 64,
                                               None) == WS
+
+
+def test_route_backward_validates_on_the_host(dl):
+    lib = dl.lib()
+    fake = ctypes.c_void_p(0x10000)
+    odd = ctypes.c_void_p(0x10002)
+    INV, UNS = 1, 2
+    assert lib.do_route_backward(None, fake, fake, 64, 8, 2, 1, 0, 0, fake, None, None) == INV
+    assert lib.do_route_backward(fake, None, fake, 64, 8, 2, 1, 0, 0, fake, None, None) == INV
+    assert lib.do_route_backward(fake, fake, None, 64, 8, 2, 1, 0, 0, fake, None, None) == INV
+    assert lib.do_route_backward(fake, fake, fake, 64, 8, 2, 1, 0, 0, None, None, None) == INV
+    assert lib.do_route_backward(fake, fake, fake, 64, 8, 2, 1, 2, 0, fake, None, None) == INV  # gate
+    assert lib.do_route_backward(fake, fake, fake, 64, 8, 2, 1, 0, 2, fake, None, None) == INV  # accumulate
+    assert lib.do_route_backward(fake, fake, fake, 64, 8, 9, 1, 0, 0, fake, None, None) == INV  # k > E
+    assert lib.do_route_backward(fake, odd, fake, 64, 8, 2, 1, 0, 0, fake, None, None) == INV
+    assert lib.do_route_backward(fake, fake, fake, 64, 8, 2, 1, 0, 0, fake, odd, None) == INV
+    assert lib.do_route_backward(fake, fake, fake, 64, 2048, 2, 1, 0, 0, fake, None, None) == UNS
