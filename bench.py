@@ -434,6 +434,36 @@ def run_ours(args, rank, world, local):
         dlogits=sets[r % N_SETS][1].dlogits, accumulate=True, status_flags=rb_flags))
     if int(rb_flags[0]) != 0:
         raise RuntimeError("do_route_backward flagged an expert id out of range")
+    # A training step's routed DO-loss split where the step splits: the forward
+    # half (routing outputs, D) and the backward half (loss, DO gradient and
+    # the combine weights' gradient in one kernel), against the one-call routed
+    # step followed by the separate routing-gradient kernel.
+    for r in range(2 * N_SETS):
+        dl.routed_forward(sets[r % N_SETS][0], k, w.gate, out=sets[r % N_SETS][1],
+                          route=routes[r % N_SETS])
+        dl.routed_backward(sets[r % N_SETS][0], routes[r % N_SETS].expert_ids, gqs[r % N_SETS], k,
+                           w.gate, 1.0, out=sets[r % N_SETS][1])
+    torch.cuda.synchronize()
+    split_fwd_ms = time_calls(lambda r: dl.routed_forward(
+        sets[r % N_SETS][0], k, w.gate, out=sets[r % N_SETS][1], route=routes[r % N_SETS]))
+
+    def split_step(r):
+        dl.routed_forward(sets[r % N_SETS][0], k, w.gate, out=sets[r % N_SETS][1],
+                          route=routes[r % N_SETS])
+        dl.routed_backward(sets[r % N_SETS][0], routes[r % N_SETS].expert_ids, gqs[r % N_SETS], k,
+                           w.gate, 1.0, out=sets[r % N_SETS][1])
+    split_ms = time_calls(split_step)
+
+    def one_call_step(r):
+        dl.forward_backward_routed(sets[r % N_SETS][0], k, w.gate, 1.0, out=sets[r % N_SETS][1],
+                                   route=routes[r % N_SETS])
+        dl.route_backward(sets[r % N_SETS][0], routes[r % N_SETS].expert_ids, gqs[r % N_SETS],
+                          w.gate, dlogits=sets[r % N_SETS][1].dlogits, accumulate=True)
+    one_call_ms = time_calls(one_call_step)
+    for r in range(N_SETS):
+        st = dl.device_status(sets[r][1].workspace)
+        if st != 0:
+            raise RuntimeError(f"device status after the split runs: {dl.status_string(st)}")
     # Context for the fractions at this size: a plain device copy of one
     # logits-sized buffer into another, in the same rotation of input sets
     # (the measured peak comes from gigabyte-sized copies).
@@ -606,6 +636,12 @@ def run_ours(args, rank, world, local):
                                  "algorithmic_bytes_accumulate":
                                      route_backward_bytes(T, E, k, L, accumulate=True),
                                  "traffic": profiled_traffic("do_route_backward")}},
+                "training_split": {
+                    "entries": "do_routed_forward then do_routed_backward (routing gradient in "
+                               "the loss kernel's epilogue)",
+                    "us_per_step": split_ms * 1e3, "forward_us": split_fwd_ms * 1e3,
+                    "vs": "do_forward_backward_routed then do_route_backward (accumulate)",
+                    "vs_us_per_step": one_call_ms * 1e3},
                 "reps": reps},
             "router_fused": {
                 "entry": "do_router_forward_backward (logits = X W^T on tcgen05 with the signature "

@@ -163,6 +163,49 @@ do_status do_routing(const float *logits, int64_t T, int32_t E, int32_t k, int32
 
 size_t do_routing_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L);
 
+/* The routed step split at the point where a training step splits it: the
+ * forward half runs when the router's outputs are needed, the backward half
+ * once the gradient of the combine weights has come back from the experts.
+ *
+ * do_routed_forward: steps 1-2 and the routing outputs from one selection
+ * pass -- bits, counts, D, origin_do (may be NULL) as do_forward_backward
+ * writes them, and expert_ids, combine and the dispatch arrays as do_routing
+ * writes them (expert_ids and combine required, the dispatch arrays may be
+ * NULL).  No loss and no gradient.
+ *
+ * do_routed_backward: step 3 on the same tokens plus the routing gradient:
+ *   loss     [L] fp32, L_DO as do_forward_backward computes it
+ *   dlogits  [L][T][E] fp32, overwritten with grad_scale * dL_DO/dz plus
+ *            the gradient of the combine weights for grad_combine [L][T][k]
+ *            (fp32) with the selection expert_ids [L][T][k] held fixed, as
+ *            do_route_backward computes it (grad_scale does not apply to it)
+ * logits, bits, counts and D are those of the forward half, expert_ids the
+ * ids it wrote.  With E = 128, the sigmoid-normalised gate, k in {1, 2, 4, 8},
+ * T <= 66052 and 16-byte aligned logits, D, bits, dlogits, expert_ids and
+ * grad_combine, the routing gradient is added in the tensor-core loss
+ * kernel's epilogue (one launch); elsewhere a second kernel adds it.  The
+ * result agrees with do_forward_backward's dlogits plus do_route_backward's
+ * within the sum of their tolerances.
+ *
+ * Both take the same workspace (do_routed_workspace_size bytes, 256-byte
+ * aligned, zero-filled before its first use): the forward half leaves in it
+ * the selected experts and the image of D that the backward half reads, so a
+ * backward call uses the workspace of the forward call on the same logits,
+ * with no other call on that workspace in between.  The backward half may be
+ * repeated.  An expert id outside [0, E) is left out and recorded in the
+ * status word (do_device_status then returns DO_ERR_INVALID_ARG).
+ * Asynchronous on `stream`. */
+do_status do_routed_forward(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
+                            int32_t gate, uint32_t *bits, int32_t *counts, int32_t *D,
+                            int64_t *origin_do, int32_t *expert_ids, float *combine,
+                            int32_t *expert_offsets, int32_t *dispatch_rows, int32_t *dispatch_pos,
+                            void *workspace, size_t workspace_bytes, void *stream);
+do_status do_routed_backward(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
+                             int32_t gate, float grad_scale, const uint32_t *bits,
+                             const int32_t *counts, const int32_t *D, const int32_t *expert_ids,
+                             const float *grad_combine, float *loss, float *dlogits,
+                             void *workspace, size_t workspace_bytes, void *stream);
+
 /* Backward of the combine weights of do_routing (Sec. 3.1.1) to the logits,
  * the selection held fixed.  With g = grad_combine, dot_t = sum_q g_tq w_tq
  * and l = expert_ids[t][q] a chosen expert:
@@ -245,13 +288,15 @@ size_t do_router_backward_workspace_size(int64_t T, int32_t E, int32_t H, int32_
 
 /* Device workspace, in bytes, that do_loss_fwd_bwd, do_forward_backward and
  * do_router_forward_backward need for these sizes (0 if the sizes are
- * invalid); do_forward_backward_routed needs do_routed_workspace_size. */
+ * invalid); do_forward_backward_routed, do_routed_forward and
+ * do_routed_backward need do_routed_workspace_size. */
 size_t do_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L);
 size_t do_routed_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L);
 
 /* Synchronizes `stream`, then reads and clears the device-side status that
- * the previous calls with this workspace recorded: DO_OK, DO_ERR_OVERFLOW or
- * DO_ERR_TIMEOUT (outputs of the failing call are then undefined). */
+ * the previous calls with this workspace recorded: DO_OK, DO_ERR_OVERFLOW,
+ * DO_ERR_TIMEOUT (outputs of the failing call are then undefined) or, after
+ * do_routed_backward, DO_ERR_INVALID_ARG for an expert id outside [0, E). */
 do_status do_device_status(void *workspace, void *stream);
 
 /* Host-to-host convenience over do_forward_backward: copies h_logits [L][T][E]

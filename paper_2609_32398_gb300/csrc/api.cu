@@ -330,6 +330,135 @@ do_status do_router_forward_backward(const void *X, const void *Wr, int64_t T, i
                                  nullptr, nullptr, &rin);
 }
 
+// The forward and backward halves of the routed step.  The forward half
+// leaves in the workspace what the backward half's loss kernel reads (the
+// selected indices, the fp16 image of D'), so the two must agree on the path;
+// the choice depends only on the logits, bits and D pointers and the shape,
+// which both halves receive.
+bool split_fast(const Problem &p, const float *logits, const uint32_t *bits, const int *D) {
+    return dol::signatures_fast_supported(logits, p) &&
+           dol::loss_fast_supported(p, logits, D, nullptr) && aligned(bits, 16);
+}
+
+// Whether the forward half writes the fp16 image of D' for the tensor-core
+// loss kernel (dlogits is not known there: the logits' alignment stands in).
+bool split_mma(const Problem &p, int gate, const float *logits, const int *D) {
+    return !alu_loss_requested() && dol::loss_mma_supported(p, gate, logits, D, logits);
+}
+
+do_status do_routed_forward(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
+                            int32_t gate, uint32_t *bits, int32_t *counts, int32_t *D,
+                            int64_t *origin_do, int32_t *expert_ids, float *combine,
+                            int32_t *expert_offsets, int32_t *dispatch_rows, int32_t *dispatch_pos,
+                            void *workspace, size_t workspace_bytes, void *stream) {
+    NvtxRange nvtx("do_routed_forward");
+    Problem p;
+    do_status st = check_sizes(T, E, k, L, &p);
+    if (st != DO_OK) return st;
+    if (!logits || !bits || !counts || !D) return DO_ERR_INVALID_ARG;
+    if (gate != DO_GATE_SIGMOID_NORM && gate != DO_GATE_SOFTMAX) return DO_ERR_INVALID_ARG;
+    if (!aligned(logits, 4) || !aligned(bits, 4) || !aligned(counts, 4) || !aligned(D, 4) ||
+        (origin_do && !aligned(origin_do, 8)))
+        return DO_ERR_INVALID_ARG;
+    const RouteArgs ra = {expert_ids, combine, expert_offsets, dispatch_rows, dispatch_pos};
+    if ((st = check_route(p, ra)) != DO_OK) return st;
+    if (!workspace || !aligned(workspace, 256) || workspace_bytes < dol::workspace_bytes(p))
+        return DO_ERR_WORKSPACE;
+    cudaStream_t s = (cudaStream_t)stream;
+    char *ws = static_cast<char *>(workspace);
+    const dol::WsLayout w = dol::ws_layout(p);
+    int *rscratch = reinterpret_cast<int *>(ws + w.route_base);
+    const dol::RouteOut route = {expert_ids, combine, gate};
+    cudaError_t e = cudaSuccess;
+    if (split_fast(p, logits, bits, D)) {
+        int *done = reinterpret_cast<int *>(ws + w.done);
+        uint8_t *idx = reinterpret_cast<uint8_t *>(ws + w.idx);
+        uint32_t *parts = reinterpret_cast<uint32_t *>(ws + w.cooc_parts);
+        int *n_acc = reinterpret_cast<int *>(ws + w.n_acc);
+        int *status = reinterpret_cast<int *>(ws);
+        const dol::ZeroSpans zero = {{done, reinterpret_cast<int *>(origin_do), nullptr},
+                                     {(int64_t)p.L, origin_do ? 2 * (int64_t)p.L : 0, 0}};
+        unsigned char *bimg =
+            split_mma(p, gate, logits, D) ? reinterpret_cast<unsigned char *>(ws + w.bimg) : nullptr;
+        if (!route_fast_ok(&ra))  // unaligned routing outputs: from the generic selection
+            e = dol::launch_signatures(logits, p, bits, counts, s, route);
+        if (e == cudaSuccess)
+            e = route_fast_ok(&ra)
+                    ? dol::launch_signatures_fast_routed(logits, p, bits, n_acc, idx, parts, zero,
+                                                         status, route, s)
+                    : dol::launch_signatures_fast(logits, p, bits, n_acc, idx, parts, zero, status, s);
+        if (e == cudaSuccess)
+            e = dol::launch_cooc_reduce(parts, dol::sig_fast_ctas_per_problem(p), n_acc, p, D,
+                                        counts, bimg, reinterpret_cast<long long *>(origin_do), s);
+        // no loss kernel follows in this call: the dispatch kernels clear the
+        // counts accumulator
+        if (e == cudaSuccess)
+            e = dol::launch_route_dispatch(bits, expert_ids, p, expert_offsets, dispatch_rows,
+                                           dispatch_pos, rscratch, s, n_acc);
+        return from_cuda(e);
+    } else {
+        e = dol::launch_signatures(logits, p, bits, counts, s, route);
+        if (e == cudaSuccess) e = dol::launch_hamming(bits, p, D, s);
+        if (e == cudaSuccess && origin_do)
+            e = dol::launch_origin_do(D, p, reinterpret_cast<long long *>(origin_do), s);
+    }
+    if (e == cudaSuccess)
+        e = dol::launch_route_dispatch(bits, expert_ids, p, expert_offsets, dispatch_rows,
+                                       dispatch_pos, rscratch, s);
+    return from_cuda(e);
+}
+
+do_status do_routed_backward(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
+                             int32_t gate, float grad_scale, const uint32_t *bits,
+                             const int32_t *counts, const int32_t *D, const int32_t *expert_ids,
+                             const float *grad_combine, float *loss, float *dlogits,
+                             void *workspace, size_t workspace_bytes, void *stream) {
+    NvtxRange nvtx("do_routed_backward");
+    Problem p;
+    do_status st = check_sizes(T, E, k, L, &p);
+    if (st != DO_OK) return st;
+    if (!logits || !bits || !counts || !D || !expert_ids || !grad_combine || !loss || !dlogits)
+        return DO_ERR_INVALID_ARG;
+    if (gate != DO_GATE_SIGMOID_NORM && gate != DO_GATE_SOFTMAX) return DO_ERR_INVALID_ARG;
+    if (!(grad_scale == grad_scale)) return DO_ERR_INVALID_ARG;
+    if (!aligned(logits, 4) || !aligned(bits, 4) || !aligned(counts, 4) || !aligned(D, 4) ||
+        !aligned(expert_ids, 4) || !aligned(grad_combine, 4) || !aligned(loss, 4) ||
+        !aligned(dlogits, 4))
+        return DO_ERR_INVALID_ARG;
+    if (!workspace || !aligned(workspace, 256) || workspace_bytes < dol::workspace_bytes(p))
+        return DO_ERR_WORKSPACE;
+    cudaStream_t s = (cudaStream_t)stream;
+    char *ws = static_cast<char *>(workspace);
+    const dol::WsLayout w = dol::ws_layout(p);
+    int *status = reinterpret_cast<int *>(ws);
+    int *done = reinterpret_cast<int *>(ws + w.done);
+    uint8_t *idx = reinterpret_cast<uint8_t *>(ws + w.idx);
+    int *n_acc = reinterpret_cast<int *>(ws + w.n_acc);
+    double *partials = reinterpret_cast<double *>(ws + w.partials);
+    cudaError_t e;
+    if (split_fast(p, logits, bits, D) && aligned(dlogits, 16)) {
+        if (split_mma(p, gate, logits, D) &&
+            dol::loss_mma_supported(p, gate, logits, D, dlogits) && aligned(expert_ids, 16) &&
+            aligned(grad_combine, 16)) {
+            // the routing gradient is added in the loss kernel's epilogue
+            return from_cuda(dol::launch_loss_mma(
+                logits, idx, reinterpret_cast<unsigned char *>(ws + w.bimg), n_acc, p, 1.0f,
+                grad_scale, loss, dlogits, partials, done, status, nullptr, s, expert_ids,
+                grad_combine));
+        }
+        e = dol::launch_loss_fast(logits, idx, D, counts, n_acc, p, gate, 1.0f, grad_scale, loss,
+                                  nullptr, dlogits, partials, done, status, nullptr, s);
+    } else {
+        e = dol::launch_loss(logits, bits, D, p, gate, 1.0f, grad_scale, loss, nullptr, dlogits,
+                             workspace, s);
+    }
+    // elsewhere the routing gradient is added by its own kernel
+    if (e == cudaSuccess)
+        e = dol::launch_route_backward(logits, expert_ids, grad_combine, p.T * p.L, E, k, gate, 1,
+                                       dlogits, status, s);
+    return from_cuda(e);
+}
+
 do_status do_routing(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L, int32_t gate,
                      int32_t *expert_ids, float *combine, int32_t *counts,
                      int32_t *expert_offsets, int32_t *dispatch_rows, int32_t *dispatch_pos,
@@ -412,6 +541,7 @@ do_status do_device_status(void *workspace, void *stream) {
     if (e != cudaSuccess) return DO_ERR_CUDA;
     if (flags & dol::kDevTimeout) return DO_ERR_TIMEOUT;
     if (flags & dol::kDevOverflow) return DO_ERR_OVERFLOW;
+    if (flags & dol::kDevBadId) return DO_ERR_INVALID_ARG;
     return DO_OK;
 }
 

@@ -15,6 +15,7 @@ constexpr unsigned kFull = 0xffffffffu;
 // Bits of the device status word kept at the start of the workspace.
 constexpr int kDevOverflow = 1;  // a row sum of D did not fit int32
 constexpr int kDevTimeout = 2;   // a bounded device wait ran out
+constexpr int kDevBadId = 4;     // an expert id given to a backward call was outside [0, E)
 
 // Workspace layout: [status word | pad to 256 B | fp64 loss partials [L][P]].
 constexpr size_t kWsHeader = 256;
@@ -61,7 +62,7 @@ struct ZeroSpans {
 };
 
 // Workspace of the loss step, carved from the caller's buffer:
-//   [0, 256)        device status word (kDevOverflow | kDevTimeout bits)
+//   [0, 256)        device status word (kDevOverflow | kDevTimeout | kDevBadId bits)
 //   done            [L] int, per-problem count of finished loss CTAs
 //   partials        [L][max CTAs per problem] fp64 sums of A_t
 //   idx             [L][T][k] uint8, the selected experts of every token
@@ -94,6 +95,7 @@ cudaError_t launch_signatures(const float *logits, const Problem &p, uint32_t *b
 cudaError_t launch_hamming(const uint32_t *bits, const Problem &p, int *D, cudaStream_t s);
 cudaError_t launch_hamming_accumulate(const uint32_t *bits, const Problem &p, int *D, int *counts,
                                       cudaStream_t s);
+cudaError_t launch_origin_do(const int *D, const Problem &p, long long *origin_do, cudaStream_t s);
 cudaError_t launch_loss(const float *logits, const uint32_t *bits, const int *D,
                         const Problem &p, int gate, float d_scale, float grad_scale,
                         float *loss, long long *origin_do, float *dlogits, void *workspace,
@@ -121,9 +123,11 @@ cudaError_t launch_route_backward(const float *z, const int32_t *ids, const floa
                                   int32_t E, int32_t k, int32_t gate, int32_t accumulate,
                                   float *dz, int32_t *status_flags, cudaStream_t s);
 
+// n_zero (may be null): an [L][E] accumulator cleared once the kernels before
+// these have finished (the scan kernel does it after its dependency wait).
 cudaError_t launch_route_dispatch(const uint32_t *bits, const int *ids, const Problem &p,
                                   int *offsets, int *rows, int *pos, int *scratch,
-                                  cudaStream_t s);
+                                  cudaStream_t s, int *n_zero = nullptr);
 // Router-side fusion (E = 128, k in {1,2,4,8}, H a multiple of 64, 16-byte
 // aligned X, W and logits): logits = X W^T on the tensor cores with the
 // fused path's signature step in the epilogue (bits, selected indices,
@@ -149,7 +153,8 @@ int loss_mma_ctas_per_problem(const Problem &p);
 cudaError_t launch_loss_mma(const float *logits, const uint8_t *idx, const unsigned char *bimg,
                             int *n_zero, const Problem &p, float d_scale, float grad_scale,
                             float *loss, float *dlogits, double *partials, int *done, int *status,
-                            int *status_out, cudaStream_t s);
+                            int *status_out, cudaStream_t s, const int *rg_ids = nullptr,
+                            const float *rg_g = nullptr);
 cudaError_t launch_loss_fast(const float *logits, const uint8_t *idx, const int *D,
                              const int *counts, int *n_zero, const Problem &p, int gate,
                              float d_scale, float grad_scale, float *loss, long long *origin_do,

@@ -191,6 +191,28 @@ loss_finalize_kernel(const double *__restrict__ partials, int P, const int *__re
     }
 }
 
+// origin_do alone (Eq. origin_do), one CTA per problem, exact in int64.
+__global__ void __launch_bounds__(256)
+origin_do_kernel(const int *__restrict__ Dg, int E, long long *__restrict__ origin_do) {
+    __shared__ long long s_red[256];
+    const int *Dl = Dg + (int64_t)blockIdx.x * E * E;
+    long long acc = 0;
+    for (int64_t idx = threadIdx.x; idx < (int64_t)E * E; idx += blockDim.x) {
+        const int i = (int)(idx / E), j = (int)(idx % E);
+        if (i != j) {
+            const long long d = Dl[idx];
+            acc += d * d;
+        }
+    }
+    s_red[threadIdx.x] = acc;
+    __syncthreads();
+    for (int o = blockDim.x / 2; o > 0; o >>= 1) {
+        if (threadIdx.x < o) s_red[threadIdx.x] += s_red[threadIdx.x + o];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) origin_do[blockIdx.x] = s_red[0];
+}
+
 template <int R, bool kSmemD, int kGate>
 cudaError_t run_loss(const float *logits, const uint32_t *bits, const int *D, const Problem &p,
                      float coef, float *dlogits, double *partials, int P, int *status,
@@ -281,6 +303,11 @@ cudaError_t launch_loss(const float *logits, const uint32_t *bits, const int *D,
     if (e != cudaSuccess) return e;
     loss_finalize_kernel<<<p.L, 256, 0, s>>>(partials, P, D, p.E, (double)d_scale * norm, loss,
                                              origin_do);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_origin_do(const int *D, const Problem &p, long long *origin_do, cudaStream_t s) {
+    origin_do_kernel<<<p.L, 256, 0, s>>>(D, p.E, origin_do);
     return cudaGetLastError();
 }
 

@@ -38,6 +38,16 @@
 //                logits of the tile after next.
 // Tensor maps are 3-D [L][T][E]: rows past the end of a problem read as zero
 // and are dropped on store.
+//
+// With the routing gradient (kRG, the backward half of the routed step), each
+// epilogue thread also adds, for its token, the gradient of the re-normalized
+// combine weights (Sec. 3.1.1) w_q = s_q / sum of the chosen s, for the
+// upstream gradient g_q of the chosen experts e_q held fixed:
+//   dz_{e_q} += w_q (1 - s_q) (g_q - sum_q' g_q' w_q').
+// The chosen logits are read from the boxes after pass 1 (each warp those in
+// its 64 columns), the two warps of the token swap their partial sums with the
+// (S, SV) exchange, and after pass 2 each adds its entries into the dz boxes
+// before the TMA store.  The sigmoid is pass 1's: one ex2 and one rcp.
 #include <cuda_fp16.h>
 
 #include <climits>
@@ -86,6 +96,15 @@ __device__ __forceinline__ float rcp_approx(float x) {
     return y;
 }
 
+// s = sigmoid(z) and 1 - s, each without cancellation, from e = 2^(-|z| log2 e)
+// and one approximate reciprocal (as pass 1 forms s)
+__device__ __forceinline__ void sigmoid_pair(float z, float &s, float &oms) {
+    const float e = ex2_approx(fabsf(z) * -kLog2e);
+    const float r = rcp_approx(1.0f + e);
+    s = z >= 0.0f ? r : e * r;
+    oms = z >= 0.0f ? e * r : r;
+}
+
 __device__ __forceinline__ int atom_add_acq_rel(int *p, int v) {
     int old;
     asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
@@ -110,7 +129,34 @@ struct MmaArgs {
     float *loss;
     int *status;
     int *status_out;  // may be null: the last CTA ORs the status word into it
+    // routing gradient (kRG): the chosen experts [L][T][K] and the upstream
+    // gradient of their combine weights [L][T][K]
+    const int *rg_ids;
+    const float *rg_g;
 };
+
+// K ints and K floats of one token row (16-, 8- or 4-byte loads)
+template <int K>
+__device__ __forceinline__ void load_route_row(const int *ids, const float *g, int (&e)[K],
+                                               float (&v)[K]) {
+    if constexpr (K >= 4) {
+#pragma unroll
+        for (int q = 0; q < K; q += 4) {
+            const int4 a = __ldg(reinterpret_cast<const int4 *>(ids + q));
+            const float4 b = __ldg(reinterpret_cast<const float4 *>(g + q));
+            e[q] = a.x; e[q + 1] = a.y; e[q + 2] = a.z; e[q + 3] = a.w;
+            v[q] = b.x; v[q + 1] = b.y; v[q + 2] = b.z; v[q + 3] = b.w;
+        }
+    } else if constexpr (K == 2) {
+        const int2 a = __ldg(reinterpret_cast<const int2 *>(ids));
+        const float2 b = __ldg(reinterpret_cast<const float2 *>(g));
+        e[0] = a.x; e[1] = a.y;
+        v[0] = b.x; v[1] = b.y;
+    } else {
+        e[0] = __ldg(ids);
+        v[0] = __ldg(g);
+    }
+}
 
 template <int K>
 __device__ __forceinline__ void load_sel(const uint8_t *p, uint32_t (&r)[2]) {
@@ -128,7 +174,7 @@ __device__ __forceinline__ void load_sel(const uint8_t *p, uint32_t (&r)[2]) {
     }
 }
 
-template <int K>
+template <int K, bool kRG>
 __global__ void __launch_bounds__(kThreads, 1)
 loss_mma_kernel(const __grid_constant__ CUtensorMap zmap, const __grid_constant__ CUtensorMap dzmap,
                 const MmaArgs a) {
@@ -312,6 +358,16 @@ loss_mma_kernel(const __grid_constant__ CUtensorMap zmap, const __grid_constant_
             ok = __all_sync(kFull, ok && !*s_abort);
             tc_fence_after();
             float S = 0.f, SV = 0.f;
+            const int64_t tok = (int64_t)(tb + m) * kTileM + row;
+            const int64_t rg_off = ((int64_t)layer * T + tok) * K;
+            // the routing inputs of this token are brought into L2 now and
+            // loaded after pass 1 (registers are full during it)
+            if constexpr (kRG) {
+                if (ok && tok < T) {
+                    asm volatile("prefetch.global.L2 [%0];" ::"l"(a.rg_ids + rg_off));
+                    asm volatile("prefetch.global.L2 [%0];" ::"l"(a.rg_g + rg_off));
+                }
+            }
             if (ok) {
                 // pass 1: s, S, SV; s (1 - s) and V back into the accumulator
 #pragma unroll 1
@@ -367,27 +423,95 @@ loss_mma_kernel(const __grid_constant__ CUtensorMap zmap, const __grid_constant_
                 }
                 tmem_wait_st();
             }
+            // Routing gradient, part 1: over the chosen experts in this warp's
+            // 64 columns, read while their logits are still in the boxes (the
+            // exchange below overwrites two 16-byte chunks of a row), the sums
+            // of their sigmoids and of g times them.  (Unshifted: this kernel
+            // already needs sum_i s_i > 0, i.e. the largest logit above about
+            // -87, and the chosen experts hold the largest logits.)
+            float zq[K];
+            float rsr = 0.0f, rsg = 0.0f;
+            bool bad_id = false;
+            int rid[K];
+            float rgv[K];
+            if constexpr (kRG) {
+                if (ok && tok < T) {
+                    load_route_row<K>(a.rg_ids + rg_off, a.rg_g + rg_off, rid, rgv);
+                } else {
+#pragma unroll
+                    for (int q = 0; q < K; ++q) { rid[q] = -1; rgv[q] = 0.0f; }
+                }
+#pragma unroll
+                for (int q = 0; q < K; ++q) {
+                    const int e = rid[q];
+                    if (tok < T && (unsigned)e >= (unsigned)kE) bad_id = true;
+                    const bool mine = (unsigned)e < (unsigned)kE && (e >> 6) == pair;
+                    zq[q] = mine ? *reinterpret_cast<const float *>(
+                                       sZ + (size_t)(group * kEpiWarps + (e >> 5) * 4 + quad) * kBoxBytes +
+                                       lane * 128 + ((((e & 31) >> 2) ^ (lane & 7)) << 4) + 4 * (e & 3))
+                                 : -INFINITY;
+                    if (mine) {
+                        float sq, omq;
+                        sigmoid_pair(zq[q], sq, omq);
+                        rsr += sq;
+                        rsg = fmaf(rgv[q], sq, rsg);
+                    }
+                }
+            }
             // exchange with the other chunk pair of the quadrant through the
-            // first 16 bytes of this row of the pair's first box
+            // first 16 bytes of this row of the pair's first box (and the next
+            // 16 for the routing gradient)
             unsigned char *myrow = sZ + (size_t)box_id(0) * kBoxBytes + lane * 128;
             float *slot = reinterpret_cast<float *>(myrow + ((lane & 7) << 4));
             slot[0] = S;
             slot[1] = SV;
             slot[2] = ok ? 1.0f : 0.0f;
+            if constexpr (kRG) {
+                slot[3] = rsr;
+                float *slot2 = reinterpret_cast<float *>(myrow + (((lane & 7) ^ 1) << 4));
+                slot2[0] = rsg;
+            }
             named_sync(1 + 4 * group + quad, 64);
             float St = 0.f, SVt = 0.f;
             bool all_ok = true;
+            float psr[2], psg[2];
 #pragma unroll
             for (int pp = 0; pp < 2; ++pp) {
-                const float *o = reinterpret_cast<const float *>(
-                    sZ + (size_t)(group * kEpiWarps + (2 * pp) * 4 + quad) * kBoxBytes + lane * 128 +
-                    ((lane & 7) << 4));
+                const unsigned char *orow =
+                    sZ + (size_t)(group * kEpiWarps + (2 * pp) * 4 + quad) * kBoxBytes + lane * 128;
+                const float *o = reinterpret_cast<const float *>(orow + ((lane & 7) << 4));
                 St += o[0];
                 SVt += o[1];
                 all_ok = all_ok && o[2] != 0.0f;
+                if constexpr (kRG) {
+                    const float *o2 = reinterpret_cast<const float *>(orow + (((lane & 7) ^ 1) << 4));
+                    psr[pp] = o[3];
+                    psg[pp] = o2[0];
+                }
             }
             all_ok = __all_sync(kFull, all_ok);
             if (!all_ok) break;  // the same decision in both warps of the quadrant
+            // Routing gradient, part 2: the two halves' sums added in pair
+            // order (the same numbers in both warps), then this warp's chosen
+            // entries: dz = w (1 - s) (g - dot), w = s / sum of the chosen s.
+            float rd[K];
+            uint32_t epk[(K + 3) / 4];
+            if constexpr (kRG) {
+                const float inv = 1.0f / (psr[0] + psr[1]);
+                const float dot = (psg[0] + psg[1]) * inv;
+#pragma unroll
+                for (int q = 0; q < K; ++q) {
+                    const bool mine = zq[q] > -INFINITY;
+                    float sq = 0.0f, omq = 0.0f;
+                    if (mine) sigmoid_pair(zq[q], sq, omq);
+                    rd[q] = sq * inv * (rgv[q] - dot) * omq;
+                    // this warp's chosen columns, one byte each (0xff: not this warp's)
+                    const uint32_t byte = mine ? (uint32_t)rid[q] : 0xffu;
+                    if (q % 4 == 0) epk[q / 4] = byte;
+                    else epk[q / 4] |= byte << (8 * (q % 4));
+                }
+                if (bad_id) atomicOr(a.status, kDevBadId);
+            }
             named_sync(1 + 4 * group + quad, 64);
             const float cs = a.coef / St;
             const float csA = cs * (SVt / St);
@@ -412,6 +536,18 @@ loss_mma_kernel(const __grid_constant__ CUtensorMap zmap, const __grid_constant_
                         o.w = __uint_as_float(jac[4 * q + 3]) * fmaf(-cs, __uint_as_float(vv[4 * q + 3]), csA);
                         *reinterpret_cast<float4 *>(zrow + (((4 * h + q) ^ (lane & 7)) << 4)) = o;
                     }
+                }
+            }
+            if constexpr (kRG) {
+                // the routing gradient added to this warp's chosen entries
+#pragma unroll
+                for (int q = 0; q < K; ++q) {
+                    const int e = (int)((epk[q / 4] >> (8 * (q % 4))) & 0xffu);
+                    if (e == 0xff) continue;
+                    float *dst = reinterpret_cast<float *>(
+                        sZ + (size_t)box_id((e >> 5) & 1) * kBoxBytes + lane * 128 +
+                        ((((e & 31) >> 2) ^ (lane & 7)) << 4) + 4 * (e & 3));
+                    *dst += rd[q];
                 }
             }
             // the accumulator may take the MMA of tile m + 2
@@ -491,10 +627,10 @@ int sms_now() {
     return n;
 }
 
-template <int K>
+template <int K, bool kRG>
 cudaError_t run_mma(const CUtensorMap &zmap, const CUtensorMap &dzmap, const MmaArgs &args, int gx,
                     int L, cudaStream_t s) {
-    cudaError_t e = ensure_smem_limit<loss_mma_kernel<K>>(kSmemMma);
+    cudaError_t e = ensure_smem_limit<loss_mma_kernel<K, kRG>>(kSmemMma);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)gx, (unsigned)L);
@@ -506,7 +642,7 @@ cudaError_t run_mma(const CUtensorMap &zmap, const CUtensorMap &dzmap, const Mma
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, loss_mma_kernel<K>, zmap, dzmap, args);
+    return cudaLaunchKernelEx(&cfg, loss_mma_kernel<K, kRG>, zmap, dzmap, args);
 }
 
 }  // namespace
@@ -533,7 +669,7 @@ int loss_mma_ctas_per_problem(const Problem &p) {
 cudaError_t launch_loss_mma(const float *logits, const uint8_t *idx, const unsigned char *bimg, int *n_zero, const Problem &p, float d_scale,
                             float grad_scale, float *loss, float *dlogits,
                             double *partials, int *done, int *status, int *status_out,
-                            cudaStream_t s) {
+                            cudaStream_t s, const int *rg_ids, const float *rg_g) {
     if (!bimg) return cudaErrorInvalidValue;
     CUtensorMap zmap, dzmap;
     if (!encode_tensor_map_3d_f32(&zmap, logits, (uint64_t)p.L, (uint64_t)p.T, (uint64_t)kE, 32) ||
@@ -556,11 +692,21 @@ cudaError_t launch_loss_mma(const float *logits, const uint8_t *idx, const unsig
     args.loss = loss;
     args.status = status;
     args.status_out = status_out;
+    args.rg_ids = rg_ids;
+    args.rg_g = rg_g;
+    if (rg_ids && rg_g) {
+        switch (p.k) {
+            case 1: return run_mma<1, true>(zmap, dzmap, args, gx, p.L, s);
+            case 2: return run_mma<2, true>(zmap, dzmap, args, gx, p.L, s);
+            case 4: return run_mma<4, true>(zmap, dzmap, args, gx, p.L, s);
+            default: return run_mma<8, true>(zmap, dzmap, args, gx, p.L, s);
+        }
+    }
     switch (p.k) {
-        case 1: return run_mma<1>(zmap, dzmap, args, gx, p.L, s);
-        case 2: return run_mma<2>(zmap, dzmap, args, gx, p.L, s);
-        case 4: return run_mma<4>(zmap, dzmap, args, gx, p.L, s);
-        default: return run_mma<8>(zmap, dzmap, args, gx, p.L, s);
+        case 1: return run_mma<1, false>(zmap, dzmap, args, gx, p.L, s);
+        case 2: return run_mma<2, false>(zmap, dzmap, args, gx, p.L, s);
+        case 4: return run_mma<4, false>(zmap, dzmap, args, gx, p.L, s);
+        default: return run_mma<8, false>(zmap, dzmap, args, gx, p.L, s);
     }
 }
 

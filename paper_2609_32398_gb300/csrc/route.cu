@@ -32,7 +32,7 @@ constexpr int kBatch = 8;  // independent global loads a scatter thread keeps in
 // dispatch order can be built as soon as the selection is done.
 __global__ void __launch_bounds__(kScanThreads)
 route_scan_kernel(const uint32_t *__restrict__ bits, int E, int64_t W, int lc, int64_t nchunks,
-                  int *__restrict__ chunk_base, int *__restrict__ totals) {
+                  int *__restrict__ chunk_base, int *__restrict__ totals, int *__restrict__ n_zero) {
     __shared__ int s_warp[kScanWarps];
     const int e = blockIdx.x, layer = blockIdx.y;
     const int tid = threadIdx.x, lane = tid & 31, wp = tid >> 5;
@@ -53,6 +53,8 @@ route_scan_kernel(const uint32_t *__restrict__ bits, int E, int64_t W, int lc, i
     // the signatures come from the kernel before this one
     pdl_wait();
     pdl_trigger();
+    // an accumulator the kernels before this one have read, cleared for the next call
+    if (n_zero && tid == 0) n_zero[(size_t)layer * E + e] = 0;
     int run = 0;
     int *cb = chunk_base + ((size_t)layer * E + e) * nchunks;
     for (int64_t c0 = 0; c0 < nchunks; c0 += kScanThreads) {
@@ -257,8 +259,9 @@ int64_t route_chunks(const Problem &p) {
 
 cudaError_t launch_route_dispatch(const uint32_t *bits, const int *ids, const Problem &p,
                                   int *offsets, int *rows, int *pos, int *scratch,
-                                  cudaStream_t s) {
-    if (!offsets && !rows && !pos) return cudaSuccess;
+                                  cudaStream_t s, int *n_zero) {
+    if (!offsets && !rows && !pos)
+        return n_zero ? cudaMemsetAsync(n_zero, 0, sizeof(int) * (size_t)p.L * p.E, s) : cudaSuccess;
     const int C = route_chunk_words(p);
     int lc = 0;
     while ((1 << lc) < C) ++lc;
@@ -275,7 +278,7 @@ cudaError_t launch_route_dispatch(const uint32_t *bits, const int *ids, const Pr
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     cudaError_t e = cudaLaunchKernelEx(&cfg, route_scan_kernel, bits, p.E, p.W, lc, nchunks,
-                                       chunk_base, totals);
+                                       chunk_base, totals, n_zero);
     if (e != cudaSuccess) return e;
     cfg.gridDim = dim3((unsigned)nchunks, (unsigned)p.L);
     cfg.blockDim = dim3(kScatterThreads);

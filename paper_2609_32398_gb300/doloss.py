@@ -47,6 +47,10 @@ EXPORTS = {
     "do_routing_workspace_size": (["i64", "i32", "i32", "i32"], "sz"),
     "do_route_backward": (["p", "p", "p", "i64", "i32", "i32", "i32", "i32", "i32", "p", "p", "p"],
                           "i32"),
+    "do_routed_forward": (["p", "i64", "i32", "i32", "i32", "i32", "p", "p", "p", "p", "p", "p", "p",
+                           "p", "p", "p", "sz", "p"], "i32"),
+    "do_routed_backward": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p", "p", "p", "p",
+                            "p", "p", "p", "sz", "p"], "i32"),
     "do_forward_backward_routed": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p", "p",
                                     "p", "p", "p", "p", "p", "p", "p", "p", "p", "sz", "p"], "i32"),
     "do_maxvio": (["p", "p", "i32", "i32", "i32", "p", "p", "p", "p"], "i32"),
@@ -275,6 +279,49 @@ def route_backward(logits, expert_ids, grad_combine, gate=GATE_SIGMOID_NORM,
         z.data_ptr(), ids.data_ptr(), g.data_ptr(), T, E, k, L, gate, int(bool(accumulate)),
         dlogits.data_ptr(), _ptr(status_flags), _stream(z)))
     return dlogits
+
+
+def routed_forward(logits, k, gate=GATE_SIGMOID_NORM, out: Buffers | None = None,
+                   route: Routing | None = None):
+    """do_routed_forward: steps 1-2 and the routing outputs (no loss, no
+    gradient).  Returns (Buffers, Routing); out.workspace carries what
+    routed_backward reads, so pass the same Buffers to it."""
+    z = _as3d(logits)
+    L, T, E = z.shape
+    if out is None:
+        out = Buffers(L, T, E, k, z.device, True)
+    if route is None:
+        route = Routing(L, T, E, k, z.device)
+    if out.shape != (L, T, E, k) or route.shape != (L, T, E, k):
+        raise ValueError("output buffers were made for another shape")
+    _check("do_routed_forward", lib().do_routed_forward(
+        z.data_ptr(), T, E, k, L, gate, out.bits.data_ptr(), out.counts.data_ptr(),
+        out.D.data_ptr(), out.origin_do.data_ptr(), route.expert_ids.data_ptr(),
+        route.combine.data_ptr(), _ptr(route.offsets), _ptr(route.rows), _ptr(route.pos),
+        out.workspace.data_ptr(), out.workspace.numel(), _stream(z)))
+    return out, route
+
+
+def routed_backward(logits, expert_ids, grad_combine, k, gate=GATE_SIGMOID_NORM, grad_scale=1.0,
+                    out: Buffers | None = None):
+    """do_routed_backward: the DO-loss and its gradient plus the combine
+    weights' gradient (grad_combine [L,T,k] fp32) in out.dlogits, after
+    routed_forward filled `out`.  Returns out."""
+    z = _as3d(logits)
+    L, T, E = z.shape
+    if out is None or out.shape != (L, T, E, k) or out.dlogits is None:
+        raise ValueError("routed_backward needs the Buffers of routed_forward (with dlogits)")
+    ids = expert_ids.reshape(L, T, k)
+    g = grad_combine.reshape(L, T, k)
+    if ids.dtype != torch.int32 or g.dtype != torch.float32:
+        raise ValueError("expert_ids must be int32 and grad_combine float32")
+    if not (ids.is_cuda and g.is_cuda and ids.is_contiguous() and g.is_contiguous()):
+        raise ValueError("expert_ids and grad_combine must be contiguous CUDA tensors")
+    _check("do_routed_backward", lib().do_routed_backward(
+        z.data_ptr(), T, E, k, L, gate, grad_scale, out.bits.data_ptr(), out.counts.data_ptr(),
+        out.D.data_ptr(), ids.data_ptr(), g.data_ptr(), out.loss.data_ptr(),
+        out.dlogits.data_ptr(), out.workspace.data_ptr(), out.workspace.numel(), _stream(z)))
+    return out
 
 
 def forward_backward_routed(logits, k, gate=GATE_SIGMOID_NORM, grad_scale=1.0,

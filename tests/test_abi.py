@@ -166,3 +166,33 @@ def test_route_backward_validates_on_the_host(dl):
     assert lib.do_route_backward(fake, odd, fake, 64, 8, 2, 1, 0, 0, fake, None, None) == INV
     assert lib.do_route_backward(fake, fake, fake, 64, 8, 2, 1, 0, 0, fake, odd, None) == INV
     assert lib.do_route_backward(fake, fake, fake, 64, 2048, 2, 1, 0, 0, fake, None, None) == UNS
+
+
+def test_routed_halves_validate_on_the_host(dl):
+    lib = dl.lib()
+    fake = ctypes.c_void_p(0x10000)
+    odd = ctypes.c_void_p(0x10002)
+    INV, WS = 1, 6
+    big = 1 << 30
+    f = lib.do_routed_forward
+    assert f(fake, 64, 8, 2, 1, 0, fake, fake, fake, None, None, fake, None, None, None, fake, big,
+             None) == INV                                                # no expert_ids
+    assert f(fake, 64, 8, 2, 1, 0, fake, fake, None, None, fake, fake, None, None, None, fake, big,
+             None) == INV                                                # no D
+    assert f(fake, 64, 8, 2, 1, 3, fake, fake, fake, None, fake, fake, None, None, None, fake, big,
+             None) == INV                                                # bad gate
+    assert f(fake, 64, 8, 2, 1, 0, fake, fake, fake, odd, fake, fake, None, None, None, fake, big,
+             None) == INV                                                # misaligned origin_do
+    assert f(fake, 64, 8, 2, 1, 0, fake, fake, fake, None, fake, fake, None, None, None, fake, 64,
+             None) == WS
+    b = lib.do_routed_backward
+    assert b(fake, 64, 8, 2, 1, 0, 1.0, fake, fake, fake, None, fake, fake, fake, fake, big,
+             None) == INV                                                # no expert_ids
+    assert b(fake, 64, 8, 2, 1, 0, 1.0, fake, fake, fake, fake, None, fake, fake, fake, big,
+             None) == INV                                                # no grad_combine
+    assert b(fake, 64, 8, 2, 1, 0, float("nan"), fake, fake, fake, fake, fake, fake, fake, fake, big,
+             None) == INV                                                # NaN grad_scale
+    assert b(fake, 64, 8, 2, 1, 0, 1.0, fake, fake, fake, odd, fake, fake, fake, fake, big,
+             None) == INV                                                # misaligned ids
+    assert b(fake, 64, 8, 2, 1, 0, 1.0, fake, fake, fake, fake, fake, fake, fake, fake, 64,
+             None) == WS
