@@ -478,19 +478,22 @@ do_status do_routing(const float *logits, int64_t T, int32_t E, int32_t k, int32
     uint32_t *bits = reinterpret_cast<uint32_t *>(ws + dol::kWsHeader);
     const dol::RouteOut route = {expert_ids, combine, gate};
     cudaError_t e;
+    int *rscratch = reinterpret_cast<int *>(ws + dol::kWsHeader + routing_bits_bytes(p));
     if (dol::signatures_fast_supported(logits, p) && route_fast_ok(&ra)) {
+        // the selection kernel writes no counts: the dispatch scan takes them
+        // from the signatures' popcounts (no memset between the kernels)
         const dol::ZeroSpans none = {{nullptr, nullptr, nullptr}, {0, 0, 0}};
-        e = cudaMemsetAsync(counts, 0, sizeof(int) * (size_t)p.L * p.E, s);
+        e = dol::launch_signatures_fast_routed(logits, p, bits, nullptr, nullptr, nullptr, none,
+                                               reinterpret_cast<int *>(ws), route, s);
         if (e == cudaSuccess)
-            e = dol::launch_signatures_fast_routed(logits, p, bits, counts, nullptr, nullptr, none,
-                                                   reinterpret_cast<int *>(ws), route, s);
-    } else {
-        e = dol::launch_signatures(logits, p, bits, counts, s, route);
+            e = dol::launch_route_dispatch(bits, expert_ids, p, expert_offsets, dispatch_rows,
+                                           dispatch_pos, rscratch, s, nullptr, counts);
+        return from_cuda(e);
     }
+    e = dol::launch_signatures(logits, p, bits, counts, s, route);
     if (e == cudaSuccess)
-        e = dol::launch_route_dispatch(
-            bits, expert_ids, p, expert_offsets, dispatch_rows, dispatch_pos,
-            reinterpret_cast<int *>(ws + dol::kWsHeader + routing_bits_bytes(p)), s);
+        e = dol::launch_route_dispatch(bits, expert_ids, p, expert_offsets, dispatch_rows,
+                                       dispatch_pos, rscratch, s);
     return from_cuda(e);
 }
 

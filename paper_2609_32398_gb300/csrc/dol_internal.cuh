@@ -125,9 +125,11 @@ cudaError_t launch_route_backward(const float *z, const int32_t *ids, const floa
 
 // n_zero (may be null): an [L][E] accumulator cleared once the kernels before
 // these have finished (the scan kernel does it after its dependency wait).
+// counts_out (may be null): n_e = |F_e| from the scan's popcounts.
 cudaError_t launch_route_dispatch(const uint32_t *bits, const int *ids, const Problem &p,
                                   int *offsets, int *rows, int *pos, int *scratch,
-                                  cudaStream_t s, int *n_zero = nullptr);
+                                  cudaStream_t s, int *n_zero = nullptr,
+                                  int *counts_out = nullptr);
 // Router-side fusion (E = 128, k in {1,2,4,8}, H a multiple of 64, 16-byte
 // aligned X, W and logits): logits = X W^T on the tensor cores with the
 // fused path's signature step in the epilogue (bits, selected indices,

@@ -32,7 +32,8 @@ constexpr int kBatch = 8;  // independent global loads a scatter thread keeps in
 // dispatch order can be built as soon as the selection is done.
 __global__ void __launch_bounds__(kScanThreads)
 route_scan_kernel(const uint32_t *__restrict__ bits, int E, int64_t W, int lc, int64_t nchunks,
-                  int *__restrict__ chunk_base, int *__restrict__ totals, int *__restrict__ n_zero) {
+                  int *__restrict__ chunk_base, int *__restrict__ totals, int *__restrict__ n_zero,
+                  int *__restrict__ counts_out) {
     __shared__ int s_warp[kScanWarps];
     const int e = blockIdx.x, layer = blockIdx.y;
     const int tid = threadIdx.x, lane = tid & 31, wp = tid >> 5;
@@ -79,7 +80,10 @@ route_scan_kernel(const uint32_t *__restrict__ bits, int E, int64_t W, int lc, i
         if (c < nchunks) cb[c] = run + before + x - n;
         run += total;
     }
-    if (tid == 0) totals[(size_t)layer * E + e] = run;
+    if (tid == 0) {
+        totals[(size_t)layer * E + e] = run;
+        if (counts_out) counts_out[(size_t)layer * E + e] = run;   // n_e = |F_e|
+    }
 }
 
 // Kernel 2, one CTA per (chunk of C = 2^lc signature words = 32 C tokens,
@@ -259,8 +263,8 @@ int64_t route_chunks(const Problem &p) {
 
 cudaError_t launch_route_dispatch(const uint32_t *bits, const int *ids, const Problem &p,
                                   int *offsets, int *rows, int *pos, int *scratch,
-                                  cudaStream_t s, int *n_zero) {
-    if (!offsets && !rows && !pos)
+                                  cudaStream_t s, int *n_zero, int *counts_out) {
+    if (!offsets && !rows && !pos && !counts_out)
         return n_zero ? cudaMemsetAsync(n_zero, 0, sizeof(int) * (size_t)p.L * p.E, s) : cudaSuccess;
     const int C = route_chunk_words(p);
     int lc = 0;
@@ -278,8 +282,9 @@ cudaError_t launch_route_dispatch(const uint32_t *bits, const int *ids, const Pr
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     cudaError_t e = cudaLaunchKernelEx(&cfg, route_scan_kernel, bits, p.E, p.W, lc, nchunks,
-                                       chunk_base, totals, n_zero);
+                                       chunk_base, totals, n_zero, counts_out);
     if (e != cudaSuccess) return e;
+    if (!offsets && !rows && !pos) return cudaSuccess;
     cfg.gridDim = dim3((unsigned)nchunks, (unsigned)p.L);
     cfg.blockDim = dim3(kScatterThreads);
     cfg.dynamicSmemBytes = sizeof(int) * (size_t)(2 * p.E * C + p.E);

@@ -448,7 +448,12 @@ template <int E, bool kRoute>
 cudaError_t dispatch_mode(const CUtensorMap &map, const Problem &p, uint32_t *bits, int *counts,
                           uint8_t *idx, uint32_t *cooc, const ZeroSpans &zero, int *status,
                           const RouteOut &route, cudaStream_t s) {
-    // split entry point: counts, no co-occurrence; fused path: co-occurrence
+    // split entry point: counts, no co-occurrence; fused path: co-occurrence;
+    // routing outputs alone: neither (the dispatch scan counts)
+    if constexpr (kRoute) {
+        if (!cooc && !counts)
+            return dispatch_k<E, false, false, true>(map, p, bits, counts, idx, cooc, zero, status, route, s);
+    }
     if (cooc) return dispatch_k<E, false, true, kRoute>(map, p, bits, counts, idx, cooc, zero, status, route, s);
     return dispatch_k<E, true, false, kRoute>(map, p, bits, counts, idx, cooc, zero, status, route, s);
 }
