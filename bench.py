@@ -70,6 +70,13 @@ def route_backward_bytes(T, E, k, L=1, accumulate=False):
     return L * (12 * T * k + (8 * T * k if accumulate else 4 * T * E))
 
 
+def routed_backward_bytes(T, E, k, L=1):
+    """Bytes of the backward half of the routed step: logits read and dlogits
+    written (4TE each), the ids and the upstream gradient (4Tk each), the
+    selected indices (Tk bytes) and the fp16 image of D' (4E^2)."""
+    return L * (8 * T * E + 9 * T * k + 4 * E * E)
+
+
 ROUTER_HIDDEN = 2048  # the 30BA3B router's input width (hidden size, Sec. 4.1)
 
 
@@ -97,6 +104,8 @@ UNIT_SOURCES = {
     "do_routing": ["sig_fast.cuh", "route.cu", "signatures.cu", "tma.cuh", "tma_host.cu",
                    "dol_internal.cuh", "api.cu"],
     "do_route_backward": ["route_bwd.cu", "dol_internal.cuh", "api.cu"],
+    "do_routed_backward": ["loss_mma.cu", "route_bwd.cu", "tma.cuh", "tma_host.cu",
+                           "dol_internal.cuh", "api.cu"],
     "do_router_forward_backward": ["router.cu", "sig_fast.cuh", "cooc_reduce.cu", "loss_mma.cu",
                                    "loss.cu", "tma.cuh", "tma_host.cu", "dol_internal.cuh",
                                    "api.cu"],
@@ -316,6 +325,16 @@ def run_ours(args, rank, world, local):
             def call(i):
                 dl.router_forward_backward(X, Wr, k, w.gate, 1.0, out=sets[0][1], logits=zr)
             ws = sets[0][1].workspace
+        elif args.quick_path == "split":
+            route = dl.Routing(L, T, E, k, dev)
+            gq = torch.randn(L, T, k, device=dev)
+
+            def call(i):
+                dl.routed_forward(sets[i % N_SETS][0], k, w.gate, out=sets[i % N_SETS][1],
+                                  route=route)
+                dl.routed_backward(sets[i % N_SETS][0], route.expert_ids, gq, k, w.gate, 1.0,
+                                   out=sets[i % N_SETS][1])
+            ws = sets[0][1].workspace
         elif args.quick_path == "route_bwd":
             route = dl.routing(sets[0][0], k, w.gate)
             gq = torch.randn(L, T, k, device=dev)
@@ -453,6 +472,9 @@ def run_ours(args, rank, world, local):
         dl.routed_backward(sets[r % N_SETS][0], routes[r % N_SETS].expert_ids, gqs[r % N_SETS], k,
                            w.gate, 1.0, out=sets[r % N_SETS][1])
     split_ms = time_calls(split_step)
+    split_bwd_ms = time_calls(lambda r: dl.routed_backward(
+        sets[r % N_SETS][0], routes[r % N_SETS].expert_ids, gqs[r % N_SETS], k, w.gate, 1.0,
+        out=sets[r % N_SETS][1]))
 
     def one_call_step(r):
         dl.forward_backward_routed(sets[r % N_SETS][0], k, w.gate, 1.0, out=sets[r % N_SETS][1],
@@ -640,6 +662,15 @@ def run_ours(args, rank, world, local):
                     "entries": "do_routed_forward then do_routed_backward (routing gradient in "
                                "the loss kernel's epilogue)",
                     "us_per_step": split_ms * 1e3, "forward_us": split_fwd_ms * 1e3,
+                    "backward_us": split_bwd_ms * 1e3,
+                    "backward_roofline": {
+                        "bound": "hbm", "kernel": "loss_mma_kernel<8, true>",
+                        "achieved": routed_backward_bytes(T, E, k, L) / (split_bwd_ms * 1e-3) / 1e9,
+                        "peak": peak, "unit": "GB/s",
+                        "frac": routed_backward_bytes(T, E, k, L) / (split_bwd_ms * 1e-3) / 1e9
+                        / peak, "peak_source": peak_src,
+                        "algorithmic_bytes": routed_backward_bytes(T, E, k, L),
+                        "traffic": profiled_traffic("do_routed_backward")},
                     "vs": "do_forward_backward_routed then do_route_backward (accumulate)",
                     "vs_us_per_step": one_call_ms * 1e3},
                 "reps": reps},
@@ -681,11 +712,12 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--quick", action="store_true",
                     help="run warmup+steps plain steps and exit (for profilers)")
-    ap.add_argument("--quick-path", choices=["loss", "routing", "routed", "router", "route_bwd"],
+    ap.add_argument("--quick-path", choices=["loss", "routing", "routed", "router", "route_bwd",
+                                             "split"],
                     default="loss",
                     help="entry point of --quick: do_forward_backward, do_routing, "
-                         "do_forward_backward_routed, do_router_forward_backward or "
-                         "do_route_backward")
+                         "do_forward_backward_routed, do_router_forward_backward, "
+                         "do_route_backward or do_routed_forward + do_routed_backward")
     args = ap.parse_args()
     if args.impl == "reference":
         rank = int(os.environ.get("RANK", "0"))
