@@ -495,6 +495,37 @@ def run_ours(args, rank, world, local):
             st = dl.device_status(ws)
             if st != 0:
                 raise RuntimeError(f"device status after the routing runs: {dl.status_string(st)}")
+    # Consumers of the counts (App. E, Sec. 3.2): MaxVio on the device for this
+    # layer and for a 48-layer stack of E = 256 experts (8 ranks each), and the
+    # host REM replica allocation for 8 ranks with 2 replica slots each.
+    R_ep = 8
+    er1 = (torch.arange(E, device=dev, dtype=torch.int32) // (E // R_ep)).contiguous()
+    c1 = sets[0][1].counts
+    E48, L48 = 256, 48
+    c48 = torch.randint(0, 2 * 65536 * 8 // E48, (L48, E48), device=dev, dtype=torch.int32,
+                        generator=torch.Generator(dev).manual_seed(5))
+    er48 = (torch.arange(E48, device=dev, dtype=torch.int32) // (E48 // R_ep)).contiguous()
+    mv_out = torch.empty(L48, dtype=torch.float64, device=dev)
+    lib = dl.lib()
+
+    def maxvio_call(cnt, er, E_, L_):
+        # the C entry point with preallocated outputs: launches back to back
+        st_ = lib.do_maxvio(cnt.data_ptr(), er.data_ptr(), E_, R_ep, L_, None, mv_out.data_ptr(),
+                            None, stream.cuda_stream)
+        if st_ != 0:
+            raise RuntimeError(dl.status_string(st_))
+    mv1_ms = time_calls(lambda r: maxvio_call(c1, er1, E, L))
+    mv48_ms = time_calls(lambda r: maxvio_call(c48, er48, E48, L48))
+    mv1, rank_loads = dl.maxvio(c1, er1, R_ep, with_rank_loads=True)
+    loads_h = rank_loads[0].double().cpu().numpy()
+    tokens_h = c1[0].double().cpu().numpy()
+    er_h = er1.cpu().numpy()
+    dl.rem_allocate(loads_h, tokens_h, er_h, 2)
+    n_rem = 200
+    t0 = time.perf_counter()
+    for _ in range(n_rem):
+        dl.rem_allocate(loads_h, tokens_h, er_h, 2)
+    rem_us = (time.perf_counter() - t0) / n_rem * 1e6
     # Router-side fusion: the router's linear map on the tensor cores with the
     # signature step in its epilogue, then the rest of the path.  X (256 MiB of
     # bf16 at H = 2048) is larger than L2 by itself.  Beside it, for context:
@@ -674,6 +705,11 @@ def run_ours(args, rank, world, local):
                     "vs": "do_forward_backward_routed then do_route_backward (accumulate)",
                     "vs_us_per_step": one_call_ms * 1e3},
                 "reps": reps},
+            "counts_consumers": {
+                "maxvio_us_per_call": {"E128_L1_R8": mv1_ms * 1e3, "E256_L48_R8": mv48_ms * 1e3},
+                "maxvio_c3": float(mv1[0]),
+                "rem_allocate_host_us_per_call": {"E128_R8_D2": rem_us},
+                "bound": "launch latency (a few KB per call)"},
             "router_fused": {
                 "entry": "do_router_forward_backward (logits = X W^T on tcgen05 with the signature "
                          "step in the GEMM epilogue, then the D reduction and the loss)",

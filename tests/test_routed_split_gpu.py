@@ -152,3 +152,36 @@ def test_bad_ids_are_reported(dl, T, E, k, gate):
     assert torch.isfinite(out.dlogits).all()
     dl.routed_backward(z, route.expert_ids, torch.ones(1, T, k, device="cuda"), k, gate, out=out)
     assert dl.device_status(out.workspace) == 0
+
+
+def test_split_with_unaligned_routing_outputs_and_no_dispatch(dl):
+    """expert_ids and combine 4- but not 16-byte aligned (the routing outputs
+    then come from the generic selection beside the fused path's) and no
+    dispatch arrays (the counts accumulator is then cleared by a memset):
+    the same outputs as the aligned call (the weights to their tolerance),
+    twice in a row."""
+    T, E, k, gate = 4096 + 33, 128, 8, 0
+    z = workloads.random_logits(T, E, seed=17, ties=True).cuda()
+    grad = torch.randn(1, T, k, device="cuda")
+    ref_out, ref_route = run_split(dl, z, k, gate, grad)
+    out = dl.Buffers(1, T, E, k)
+    route = dl.Routing(1, T, E, k, with_dispatch=False)
+    ids_store = torch.empty(T * k + 1, dtype=torch.int32, device="cuda")
+    comb_store = torch.empty(T * k + 1, dtype=torch.float32, device="cuda")
+    route.expert_ids = ids_store[1:].view(1, T, k)
+    route.combine = comb_store[1:].view(1, T, k)
+    for _ in range(2):
+        dl.routed_forward(z, k, gate, out=out, route=route)
+        torch.cuda.synchronize()
+        assert torch.equal(route.expert_ids, ref_route.expert_ids)
+        # the generic selection kernel sums the weights in another order:
+        # both are within 2(k + 12) 2^-24 of the exact ratio
+        assert (route.combine - ref_route.combine).abs().max() <= 4 * (k + 12) * 2.0 ** -24
+        assert torch.equal(out.counts, ref_out.counts) and torch.equal(out.D, ref_out.D)
+        assert torch.equal(out.origin_do, ref_out.origin_do)
+    ids_aligned = route.expert_ids.clone()
+    dl.routed_backward(z, ids_aligned, grad, k, gate, out=out)
+    torch.cuda.synchronize()
+    assert dl.device_status(out.workspace) == 0
+    assert torch.equal(out.loss, ref_out.loss)
+    assert torch.equal(out.dlogits, ref_out.dlogits)
