@@ -618,6 +618,45 @@ def do_loss(logits: torch.Tensor, k: int, gate=GATE_SIGMOID_NORM) -> torch.Tenso
     return _DOLossFunction.apply(_as3d(logits) if logits.dim() == 3 else logits, k, gate)
 
 
+class _RouteFunction(torch.autograd.Function):
+    """The routing outputs of one call as an autograd node: the forward runs
+    do_routing (ids, combine weights, dispatch order); the backward sends the
+    incoming gradient of the combine weights to the logits through
+    do_route_backward, the selection held fixed."""
+
+    @staticmethod
+    def forward(ctx, logits, k, gate):
+        z = _as3d(logits.detach())
+        route = routing(z, k, gate)
+        ctx.save_for_backward(z, route.expert_ids)
+        ctx.gate = gate
+        ctx.squeeze = logits.dim() == 2
+        ids, combine = route.expert_ids, route.combine
+        if ctx.squeeze:
+            ids, combine = ids[0], combine[0]
+        ctx.mark_non_differentiable(ids)
+        return ids, combine, route
+
+    @staticmethod
+    def backward(ctx, grad_ids, grad_combine, grad_route):
+        z, ids = ctx.saved_tensors
+        if grad_combine is None:
+            return None, None, None
+        g = grad_combine.reshape(ids.shape).to(torch.float32).contiguous()
+        dz = route_backward(z, ids, g, ctx.gate)
+        return (dz[0] if ctx.squeeze else dz), None, None
+
+
+def route(logits: torch.Tensor, k: int, gate=GATE_SIGMOID_NORM):
+    """Routing of router logits [T,E] or [L,T,E] (fp32, CUDA) for an MoE layer
+    (Sec. 3.1.1): returns (expert_ids, combine, Routing) where combine, the
+    re-normalized weights of the chosen experts, is differentiable -- its
+    gradient reaches the logits through autograd with the choice of experts
+    held fixed -- and the Routing also holds the counts and the dispatch
+    order."""
+    return _RouteFunction.apply(logits, k, gate)
+
+
 def offdiag_variance(origin_do, T: int, E: int, k: int):
     """Variance of the off-diagonal entries of a local Hamming matrix, from
     Eq. origin_do (the exact sum of their squares) and Eq. zero_sum (their sum

@@ -192,3 +192,27 @@ def test_do_loss_plus_routing_gradient_in_one_buffer(dl):
     got = out.dlogits[0].double().cpu().numpy()
     tol = 1e-4 * np.abs(ref_do).max() + bound(zl, ids, grad[0].cpu().numpy(), w.gate)
     assert (np.abs(got - (ref_do + ref_route)) <= tol).all()
+
+
+@pytest.mark.parametrize("gate", [0, 1])
+def test_autograd_route_with_the_do_loss(dl, gate):
+    """dl.route as an autograd node: a loss built from the combine weights and
+    the DO-loss together backpropagate to the logits as the oracle's two
+    gradients summed (combine weights: the selection held fixed)."""
+    T, E, k = 2048 + 3, 128, 8
+    z_cpu = workloads.random_logits(T, E, seed=41)[0]
+    z = z_cpu.cuda().requires_grad_(True)
+    ids, combine, route = dl.route(z, k, gate)
+    assert ids.shape == (T, k) and combine.shape == (T, k) and not ids.requires_grad
+    u = torch.randn(T, k, generator=torch.Generator().manual_seed(2)).cuda()
+    lam = 0.25
+    objective = (combine * u).sum() + lam * dl.do_loss(z, k, gate)
+    objective.backward()
+    zl = z_cpu.numpy()
+    ids_ref, _ = oracle.route(zl, k, gate)
+    assert np.array_equal(ids.cpu().numpy(), ids_ref)
+    want_route = oracle.route_backward(zl, ids_ref, u.double().cpu().numpy(), gate)
+    want_do = lam * oracle.forward_backward(zl, k, gate)["dz"]
+    tol = 1e-4 * np.abs(want_do).max() + bound(zl, ids_ref, u.cpu().numpy(), gate)
+    got = z.grad.double().cpu().numpy()
+    assert (np.abs(got - (want_route + want_do)) <= tol).all()
