@@ -36,6 +36,7 @@ WORKLOAD = "c3"
 METRIC = "DO-loss fwd+bwd routed tokens/s at E=128,k=8; % of GB300 HBM roofline"
 UNIT = "tokens/s"
 N_SETS = 8
+NOMINAL_HBM_GBS = 8000.0  # GB300 HBM3e, nominal (context for the measured-peak fraction)
 KERNELS_PER_STEP = 3  # signatures (+ co-occurrence), co-occurrence reduce (D), loss + gradient
 
 
@@ -655,7 +656,9 @@ def run_ours(args, rank, world, local):
                          "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "peak_source": peak_src,
                          "algorithmic_bytes": algorithmic_bytes(T, E, L),
-                         "traffic": profiled_traffic("do_forward_backward")},
+                         "traffic": profiled_traffic("do_forward_backward"),
+                         "frac_of_nominal_8000_GBs": achieved / NOMINAL_HBM_GBS},
+            "assignments_per_s": value * k,
             "split_entry_points": {"us": {k_: v * 1e3 for k_, v in stage_ms.items()},
                                    "GB/s": split_gbs},
             "size_matched_copy": {
