@@ -193,8 +193,10 @@ size_t do_routing_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L);
  * backward call uses the workspace of the forward call on the same logits,
  * with no other call on that workspace in between.  The backward half may be
  * repeated.  An expert id outside [0, E) is left out and recorded in the
- * status word (do_device_status then returns DO_ERR_INVALID_ARG).
- * Asynchronous on `stream`. */
+ * status word (do_device_status then returns DO_ERR_INVALID_ARG).  The loss
+ * uses the D of these tokens (d_scale = 1); a Hamming matrix summed over
+ * data-parallel ranks (Eq. global_do) goes through do_loss_fwd_bwd followed
+ * by do_route_backward instead.  Asynchronous on `stream`. */
 do_status do_routed_forward(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
                             int32_t gate, uint32_t *bits, int32_t *counts, int32_t *D,
                             int64_t *origin_do, int32_t *expert_ids, float *combine,
