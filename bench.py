@@ -477,6 +477,17 @@ def run_ours(args, rank, world, local):
         sets[r % N_SETS][0], routes[r % N_SETS].expert_ids, gqs[r % N_SETS], k, w.gate, 1.0,
         out=sets[r % N_SETS][1]))
 
+    # Global-DO's per-rank step (Sec. 3.1.4, Eq. global_do) through the halves:
+    # the local D (standing in for the matrix summed over the ranks, whose
+    # exchange is a 64 KB all-reduce between the halves) with d_scale = 1/2,
+    # which takes the ALU loss kernel; against the three split entry points.
+    def global_step(r):
+        dl.routed_forward(sets[r % N_SETS][0], k, w.gate, out=sets[r % N_SETS][1],
+                          with_routing=False)
+        dl.routed_backward(sets[r % N_SETS][0], None, None, k, w.gate, 1.0,
+                           out=sets[r % N_SETS][1], d_scale=0.5)
+    global_ms = time_calls(global_step)
+
     def one_call_step(r):
         dl.forward_backward_routed(sets[r % N_SETS][0], k, w.gate, 1.0, out=sets[r % N_SETS][1],
                                    route=routes[r % N_SETS])
@@ -692,6 +703,12 @@ def run_ours(args, rank, world, local):
                                  "algorithmic_bytes_accumulate":
                                      route_backward_bytes(T, E, k, L, accumulate=True),
                                  "traffic": profiled_traffic("do_route_backward")}},
+                "global_do_step": {
+                    "entries": "do_routed_forward (no routing outputs) then do_routed_backward "
+                               "with a summed D and d_scale = 1/2",
+                    "us_per_step": global_ms * 1e3,
+                    "vs": "do_signatures + do_pairwise_hamming + do_loss_fwd_bwd",
+                    "vs_us_per_step": sum(stage_ms.values()) * 1e3},
                 "training_split": {
                     "entries": "do_routed_forward then do_routed_backward (routing gradient in "
                                "the loss kernel's epilogue)",

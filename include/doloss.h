@@ -170,22 +170,27 @@ size_t do_routing_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L);
  * do_routed_forward: steps 1-2 and the routing outputs from one selection
  * pass -- bits, counts, D, origin_do (may be NULL) as do_forward_backward
  * writes them, and expert_ids, combine and the dispatch arrays as do_routing
- * writes them (expert_ids and combine required, the dispatch arrays may be
- * NULL).  No loss and no gradient.
+ * writes them (the dispatch arrays may be NULL; with expert_ids and combine
+ * both NULL, and no dispatch arrays, the call is steps 1-2 alone).  No loss
+ * and no gradient.
  *
  * do_routed_backward: step 3 on the same tokens plus the routing gradient:
- *   loss     [L] fp32, L_DO as do_forward_backward computes it
+ *   loss     [L] fp32, L_DO as do_loss_fwd_bwd computes it with D and d_scale
  *   dlogits  [L][T][E] fp32, overwritten with grad_scale * dL_DO/dz plus
  *            the gradient of the combine weights for grad_combine [L][T][k]
  *            (fp32) with the selection expert_ids [L][T][k] held fixed, as
- *            do_route_backward computes it (grad_scale does not apply to it)
- * logits, bits, counts and D are those of the forward half, expert_ids the
- * ids it wrote.  With E = 128, the sigmoid-normalised gate, k in {1, 2, 4, 8},
+ *            do_route_backward computes it (grad_scale does not apply to it;
+ *            expert_ids and grad_combine both NULL: no routing gradient)
+ * logits, bits and counts are those of the forward half, expert_ids the ids
+ * it wrote.  With d_scale = 1, D is the forward half's matrix; otherwise D
+ * is a matrix summed over data-parallel ranks or micro-batches that include
+ * these tokens (Eq. global_do, d_scale = 1 / their number) and m stays T.
+ * With d_scale = 1, E = 128, the sigmoid-normalised gate, k in {1, 2, 4, 8},
  * T <= 66052 and 16-byte aligned logits, D, bits, dlogits, expert_ids and
- * grad_combine, the routing gradient is added in the tensor-core loss
- * kernel's epilogue (one launch); elsewhere a second kernel adds it.  The
- * result agrees with do_forward_backward's dlogits plus do_route_backward's
- * within the sum of their tolerances.
+ * grad_combine, the tensor-core loss kernel runs and adds the routing
+ * gradient in its epilogue (one launch); elsewhere the ALU loss kernels run
+ * and a second kernel adds it.  The result agrees with do_loss_fwd_bwd's
+ * dlogits plus do_route_backward's within the sum of their tolerances.
  *
  * Both take the same workspace (do_routed_workspace_size bytes, 256-byte
  * aligned, zero-filled before its first use): the forward half leaves in it
@@ -193,17 +198,15 @@ size_t do_routing_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L);
  * backward call uses the workspace of the forward call on the same logits,
  * with no other call on that workspace in between.  The backward half may be
  * repeated.  An expert id outside [0, E) is left out and recorded in the
- * status word (do_device_status then returns DO_ERR_INVALID_ARG).  The loss
- * uses the D of these tokens (d_scale = 1); a Hamming matrix summed over
- * data-parallel ranks (Eq. global_do) goes through do_loss_fwd_bwd followed
- * by do_route_backward instead.  Asynchronous on `stream`. */
+ * status word (do_device_status then returns DO_ERR_INVALID_ARG).
+ * Asynchronous on `stream`. */
 do_status do_routed_forward(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
                             int32_t gate, uint32_t *bits, int32_t *counts, int32_t *D,
                             int64_t *origin_do, int32_t *expert_ids, float *combine,
                             int32_t *expert_offsets, int32_t *dispatch_rows, int32_t *dispatch_pos,
                             void *workspace, size_t workspace_bytes, void *stream);
 do_status do_routed_backward(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
-                             int32_t gate, float grad_scale, const uint32_t *bits,
+                             int32_t gate, float d_scale, float grad_scale, const uint32_t *bits,
                              const int32_t *counts, const int32_t *D, const int32_t *expert_ids,
                              const float *grad_combine, float *loss, float *dlogits,
                              void *workspace, size_t workspace_bytes, void *stream);

@@ -360,8 +360,12 @@ do_status do_routed_forward(const float *logits, int64_t T, int32_t E, int32_t k
     if (!aligned(logits, 4) || !aligned(bits, 4) || !aligned(counts, 4) || !aligned(D, 4) ||
         (origin_do && !aligned(origin_do, 8)))
         return DO_ERR_INVALID_ARG;
+    // without routing outputs (expert_ids and combine both NULL, and no
+    // dispatch arrays) the call is steps 1-2 alone
+    const bool routed = expert_ids || combine;
     const RouteArgs ra = {expert_ids, combine, expert_offsets, dispatch_rows, dispatch_pos};
-    if ((st = check_route(p, ra)) != DO_OK) return st;
+    if (routed && (st = check_route(p, ra)) != DO_OK) return st;
+    if (!routed && (expert_offsets || dispatch_rows || dispatch_pos)) return DO_ERR_INVALID_ARG;
     if (!workspace || !aligned(workspace, 256) || workspace_bytes < dol::workspace_bytes(p))
         return DO_ERR_WORKSPACE;
     cudaStream_t s = (cudaStream_t)stream;
@@ -369,6 +373,7 @@ do_status do_routed_forward(const float *logits, int64_t T, int32_t E, int32_t k
     const dol::WsLayout w = dol::ws_layout(p);
     int *rscratch = reinterpret_cast<int *>(ws + w.route_base);
     const dol::RouteOut route = {expert_ids, combine, gate};
+    const RouteArgs *rap = routed ? &ra : nullptr;
     cudaError_t e = cudaSuccess;
     if (split_fast(p, logits, bits, D)) {
         int *done = reinterpret_cast<int *>(ws + w.done);
@@ -380,10 +385,10 @@ do_status do_routed_forward(const float *logits, int64_t T, int32_t E, int32_t k
                                      {(int64_t)p.L, origin_do ? 2 * (int64_t)p.L : 0, 0}};
         unsigned char *bimg =
             split_mma(p, gate, logits, D) ? reinterpret_cast<unsigned char *>(ws + w.bimg) : nullptr;
-        if (!route_fast_ok(&ra))  // unaligned routing outputs: from the generic selection
+        if (routed && !route_fast_ok(rap))  // unaligned routing outputs: the generic selection
             e = dol::launch_signatures(logits, p, bits, counts, s, route);
         if (e == cudaSuccess)
-            e = route_fast_ok(&ra)
+            e = routed && route_fast_ok(rap)
                     ? dol::launch_signatures_fast_routed(logits, p, bits, n_acc, idx, parts, zero,
                                                          status, route, s)
                     : dol::launch_signatures_fast(logits, p, bits, n_acc, idx, parts, zero, status, s);
@@ -397,7 +402,8 @@ do_status do_routed_forward(const float *logits, int64_t T, int32_t E, int32_t k
                                            dispatch_pos, rscratch, s, n_acc);
         return from_cuda(e);
     } else {
-        e = dol::launch_signatures(logits, p, bits, counts, s, route);
+        e = routed ? dol::launch_signatures(logits, p, bits, counts, s, route)
+                   : dol::launch_signatures(logits, p, bits, counts, s);
         if (e == cudaSuccess) e = dol::launch_hamming(bits, p, D, s);
         if (e == cudaSuccess && origin_do)
             e = dol::launch_origin_do(D, p, reinterpret_cast<long long *>(origin_do), s);
@@ -409,7 +415,7 @@ do_status do_routed_forward(const float *logits, int64_t T, int32_t E, int32_t k
 }
 
 do_status do_routed_backward(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
-                             int32_t gate, float grad_scale, const uint32_t *bits,
+                             int32_t gate, float d_scale, float grad_scale, const uint32_t *bits,
                              const int32_t *counts, const int32_t *D, const int32_t *expert_ids,
                              const float *grad_combine, float *loss, float *dlogits,
                              void *workspace, size_t workspace_bytes, void *stream) {
@@ -417,12 +423,14 @@ do_status do_routed_backward(const float *logits, int64_t T, int32_t E, int32_t 
     Problem p;
     do_status st = check_sizes(T, E, k, L, &p);
     if (st != DO_OK) return st;
-    if (!logits || !bits || !counts || !D || !expert_ids || !grad_combine || !loss || !dlogits)
-        return DO_ERR_INVALID_ARG;
+    if (!logits || !bits || !counts || !D || !loss || !dlogits) return DO_ERR_INVALID_ARG;
+    // the routing gradient is optional: expert_ids and grad_combine together
+    if (!expert_ids != !grad_combine) return DO_ERR_INVALID_ARG;
+    const bool rg = expert_ids != nullptr;
     if (gate != DO_GATE_SIGMOID_NORM && gate != DO_GATE_SOFTMAX) return DO_ERR_INVALID_ARG;
-    if (!(grad_scale == grad_scale)) return DO_ERR_INVALID_ARG;
+    if (!(grad_scale == grad_scale) || !(d_scale == d_scale)) return DO_ERR_INVALID_ARG;
     if (!aligned(logits, 4) || !aligned(bits, 4) || !aligned(counts, 4) || !aligned(D, 4) ||
-        !aligned(expert_ids, 4) || !aligned(grad_combine, 4) || !aligned(loss, 4) ||
+        (rg && (!aligned(expert_ids, 4) || !aligned(grad_combine, 4))) || !aligned(loss, 4) ||
         !aligned(dlogits, 4))
         return DO_ERR_INVALID_ARG;
     if (!workspace || !aligned(workspace, 256) || workspace_bytes < dol::workspace_bytes(p))
@@ -435,25 +443,31 @@ do_status do_routed_backward(const float *logits, int64_t T, int32_t E, int32_t 
     uint8_t *idx = reinterpret_cast<uint8_t *>(ws + w.idx);
     int *n_acc = reinterpret_cast<int *>(ws + w.n_acc);
     double *partials = reinterpret_cast<double *>(ws + w.partials);
+    // d_scale = 1: D is the forward half's own matrix, whose fp16 image the
+    // forward half left for the tensor-core kernel; otherwise D is a matrix
+    // summed over ranks or micro-batches (Eq. global_do), read as given.
+    const bool local = d_scale == 1.0f;
     cudaError_t e;
     if (split_fast(p, logits, bits, D) && aligned(dlogits, 16)) {
-        if (split_mma(p, gate, logits, D) &&
-            dol::loss_mma_supported(p, gate, logits, D, dlogits) && aligned(expert_ids, 16) &&
-            aligned(grad_combine, 16)) {
+        if (local && split_mma(p, gate, logits, D) &&
+            dol::loss_mma_supported(p, gate, logits, D, dlogits) &&
+            (!rg || (aligned(expert_ids, 16) && aligned(grad_combine, 16)))) {
             // the routing gradient is added in the loss kernel's epilogue
             return from_cuda(dol::launch_loss_mma(
                 logits, idx, reinterpret_cast<unsigned char *>(ws + w.bimg), n_acc, p, 1.0f,
                 grad_scale, loss, dlogits, partials, done, status, nullptr, s, expert_ids,
                 grad_combine));
         }
-        e = dol::launch_loss_fast(logits, idx, D, counts, n_acc, p, gate, 1.0f, grad_scale, loss,
-                                  nullptr, dlogits, partials, done, status, nullptr, s);
+        // the row sums of D come from the counts only for the local matrix
+        e = dol::launch_loss_fast(logits, idx, D, local ? counts : nullptr, n_acc, p, gate,
+                                  d_scale, grad_scale, loss, nullptr, dlogits, partials, done,
+                                  status, nullptr, s);
     } else {
-        e = dol::launch_loss(logits, bits, D, p, gate, 1.0f, grad_scale, loss, nullptr, dlogits,
+        e = dol::launch_loss(logits, bits, D, p, gate, d_scale, grad_scale, loss, nullptr, dlogits,
                              workspace, s);
     }
     // elsewhere the routing gradient is added by its own kernel
-    if (e == cudaSuccess)
+    if (e == cudaSuccess && rg)
         e = dol::launch_route_backward(logits, expert_ids, grad_combine, p.T * p.L, E, k, gate, 1,
                                        dlogits, status, s);
     return from_cuda(e);

@@ -49,8 +49,8 @@ EXPORTS = {
                           "i32"),
     "do_routed_forward": (["p", "i64", "i32", "i32", "i32", "i32", "p", "p", "p", "p", "p", "p", "p",
                            "p", "p", "p", "sz", "p"], "i32"),
-    "do_routed_backward": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p", "p", "p", "p",
-                            "p", "p", "p", "sz", "p"], "i32"),
+    "do_routed_backward": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "f32", "p", "p", "p", "p",
+                            "p", "p", "p", "p", "sz", "p"], "i32"),
     "do_forward_backward_routed": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "p", "p", "p",
                                     "p", "p", "p", "p", "p", "p", "p", "p", "p", "sz", "p"], "i32"),
     "do_maxvio": (["p", "p", "i32", "i32", "i32", "p", "p", "p", "p"], "i32"),
@@ -282,44 +282,57 @@ def route_backward(logits, expert_ids, grad_combine, gate=GATE_SIGMOID_NORM,
 
 
 def routed_forward(logits, k, gate=GATE_SIGMOID_NORM, out: Buffers | None = None,
-                   route: Routing | None = None):
-    """do_routed_forward: steps 1-2 and the routing outputs (no loss, no
-    gradient).  Returns (Buffers, Routing); out.workspace carries what
-    routed_backward reads, so pass the same Buffers to it."""
+                   route: Routing | None = None, with_routing=True):
+    """do_routed_forward: steps 1-2 and (with_routing) the routing outputs;
+    no loss, no gradient.  Returns (Buffers, Routing or None); out.workspace
+    carries what routed_backward reads, so pass the same Buffers to it."""
     z = _as3d(logits)
     L, T, E = z.shape
     if out is None:
         out = Buffers(L, T, E, k, z.device, True)
-    if route is None:
+    if with_routing and route is None:
         route = Routing(L, T, E, k, z.device)
-    if out.shape != (L, T, E, k) or route.shape != (L, T, E, k):
+    if not with_routing:
+        route = None
+    if out.shape != (L, T, E, k) or (route is not None and route.shape != (L, T, E, k)):
         raise ValueError("output buffers were made for another shape")
+    r = route
     _check("do_routed_forward", lib().do_routed_forward(
         z.data_ptr(), T, E, k, L, gate, out.bits.data_ptr(), out.counts.data_ptr(),
-        out.D.data_ptr(), out.origin_do.data_ptr(), route.expert_ids.data_ptr(),
-        route.combine.data_ptr(), _ptr(route.offsets), _ptr(route.rows), _ptr(route.pos),
+        out.D.data_ptr(), out.origin_do.data_ptr(), _ptr(r.expert_ids if r else None),
+        _ptr(r.combine if r else None), _ptr(r.offsets if r else None),
+        _ptr(r.rows if r else None), _ptr(r.pos if r else None),
         out.workspace.data_ptr(), out.workspace.numel(), _stream(z)))
     return out, route
 
 
 def routed_backward(logits, expert_ids, grad_combine, k, gate=GATE_SIGMOID_NORM, grad_scale=1.0,
-                    out: Buffers | None = None):
+                    out: Buffers | None = None, D: torch.Tensor | None = None, d_scale=1.0):
     """do_routed_backward: the DO-loss and its gradient plus the combine
-    weights' gradient (grad_combine [L,T,k] fp32) in out.dlogits, after
-    routed_forward filled `out`.  Returns out."""
+    weights' gradient (grad_combine [L,T,k] fp32; expert_ids and grad_combine
+    may both be None) in out.dlogits, after routed_forward filled `out`.  D
+    (default out.D) with d_scale: a matrix summed over ranks or micro-batches
+    (Eq. global_do).  Returns out."""
     z = _as3d(logits)
     L, T, E = z.shape
     if out is None or out.shape != (L, T, E, k) or out.dlogits is None:
         raise ValueError("routed_backward needs the Buffers of routed_forward (with dlogits)")
-    ids = expert_ids.reshape(L, T, k)
-    g = grad_combine.reshape(L, T, k)
-    if ids.dtype != torch.int32 or g.dtype != torch.float32:
-        raise ValueError("expert_ids must be int32 and grad_combine float32")
-    if not (ids.is_cuda and g.is_cuda and ids.is_contiguous() and g.is_contiguous()):
-        raise ValueError("expert_ids and grad_combine must be contiguous CUDA tensors")
+    if (expert_ids is None) != (grad_combine is None):
+        raise ValueError("expert_ids and grad_combine go together")
+    ids = g = None
+    if expert_ids is not None:
+        ids = expert_ids.reshape(L, T, k)
+        g = grad_combine.reshape(L, T, k)
+        if ids.dtype != torch.int32 or g.dtype != torch.float32:
+            raise ValueError("expert_ids must be int32 and grad_combine float32")
+        if not (ids.is_cuda and g.is_cuda and ids.is_contiguous() and g.is_contiguous()):
+            raise ValueError("expert_ids and grad_combine must be contiguous CUDA tensors")
+    Dm = out.D if D is None else D
+    if Dm.shape != (L, E, E) or Dm.dtype != torch.int32 or not Dm.is_contiguous():
+        raise ValueError("D must be a contiguous int32 [L,E,E] tensor")
     _check("do_routed_backward", lib().do_routed_backward(
-        z.data_ptr(), T, E, k, L, gate, grad_scale, out.bits.data_ptr(), out.counts.data_ptr(),
-        out.D.data_ptr(), ids.data_ptr(), g.data_ptr(), out.loss.data_ptr(),
+        z.data_ptr(), T, E, k, L, gate, d_scale, grad_scale, out.bits.data_ptr(),
+        out.counts.data_ptr(), Dm.data_ptr(), _ptr(ids), _ptr(g), out.loss.data_ptr(),
         out.dlogits.data_ptr(), out.workspace.data_ptr(), out.workspace.numel(), _stream(z)))
     return out
 
@@ -549,13 +562,12 @@ def global_forward_backward(logits, k, gate=GATE_SIGMOID_NORM, grad_scale=1.0, g
     gradient with d_scale = 1/ranks (m stays the local token count).
     Returns (loss [L], dlogits [L,T,E], D_global [L,E,E] int32, counts [L,E])."""
     z = _as3d(logits)
-    L, T, E = z.shape
-    bits, counts = signatures(z, k)
-    D = pairwise_hamming(bits, T)
-    D, d_scale = all_reduce_distances(D, group)
-    loss, _, dz = loss_fwd_bwd(z, bits, D, k, gate, d_scale=d_scale, grad_scale=grad_scale,
-                               with_origin=False)
-    return loss, dz, D, counts
+    # the forward half (fused selection and co-occurrence reduction), the sum
+    # over the ranks, then the backward half with that matrix
+    out, _ = routed_forward(z, k, gate, with_routing=False)
+    D, d_scale = all_reduce_distances(out.D, group)
+    routed_backward(z, None, None, k, gate, grad_scale, out=out, D=D, d_scale=d_scale)
+    return out.loss, out.dlogits, D, out.counts
 
 
 def window_forward_backward(logits_list, k, gate=GATE_SIGMOID_NORM, grad_scale=1.0, group=None):

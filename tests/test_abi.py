@@ -176,7 +176,7 @@ def test_routed_halves_validate_on_the_host(dl):
     big = 1 << 30
     f = lib.do_routed_forward
     assert f(fake, 64, 8, 2, 1, 0, fake, fake, fake, None, None, fake, None, None, None, fake, big,
-             None) == INV                                                # no expert_ids
+             None) == INV                                                # combine without ids
     assert f(fake, 64, 8, 2, 1, 0, fake, fake, None, None, fake, fake, None, None, None, fake, big,
              None) == INV                                                # no D
     assert f(fake, 64, 8, 2, 1, 3, fake, fake, fake, None, fake, fake, None, None, None, fake, big,
@@ -186,13 +186,20 @@ def test_routed_halves_validate_on_the_host(dl):
     assert f(fake, 64, 8, 2, 1, 0, fake, fake, fake, None, fake, fake, None, None, None, fake, 64,
              None) == WS
     b = lib.do_routed_backward
-    assert b(fake, 64, 8, 2, 1, 0, 1.0, fake, fake, fake, None, fake, fake, fake, fake, big,
-             None) == INV                                                # no expert_ids
-    assert b(fake, 64, 8, 2, 1, 0, 1.0, fake, fake, fake, fake, None, fake, fake, fake, big,
-             None) == INV                                                # no grad_combine
-    assert b(fake, 64, 8, 2, 1, 0, float("nan"), fake, fake, fake, fake, fake, fake, fake, fake, big,
-             None) == INV                                                # NaN grad_scale
-    assert b(fake, 64, 8, 2, 1, 0, 1.0, fake, fake, fake, odd, fake, fake, fake, fake, big,
+    assert b(fake, 64, 8, 2, 1, 0, 1.0, 1.0, fake, fake, fake, None, fake, fake, fake, fake, big,
+             None) == INV                                                # ids without gradient
+    assert b(fake, 64, 8, 2, 1, 0, 1.0, 1.0, fake, fake, fake, fake, None, fake, fake, fake, big,
+             None) == INV                                                # gradient without ids
+    assert b(fake, 64, 8, 2, 1, 0, 1.0, float("nan"), fake, fake, fake, fake, fake, fake, fake, fake,
+             big, None) == INV                                           # NaN grad_scale
+    assert b(fake, 64, 8, 2, 1, 0, float("nan"), 1.0, fake, fake, fake, fake, fake, fake, fake, fake,
+             big, None) == INV                                           # NaN d_scale
+    assert b(fake, 64, 8, 2, 1, 0, 1.0, 1.0, fake, fake, fake, odd, fake, fake, fake, fake, big,
              None) == INV                                                # misaligned ids
-    assert b(fake, 64, 8, 2, 1, 0, 1.0, fake, fake, fake, fake, fake, fake, fake, fake, 64,
+    assert b(fake, 64, 8, 2, 1, 0, 1.0, 1.0, fake, fake, None, None, None, fake, fake, fake, big,
+             None) == INV                                                # no D
+    assert b(fake, 64, 8, 2, 1, 0, 1.0, 1.0, fake, fake, fake, fake, fake, fake, fake, fake, 64,
              None) == WS
+    # steps 1-2 alone: routing outputs absent, but then no dispatch arrays either
+    assert f(fake, 64, 8, 2, 1, 0, fake, fake, fake, None, None, None, fake, None, None, fake, big,
+             None) == INV

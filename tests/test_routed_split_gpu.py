@@ -185,3 +185,51 @@ def test_split_with_unaligned_routing_outputs_and_no_dispatch(dl):
     assert dl.device_status(out.workspace) == 0
     assert torch.equal(out.loss, ref_out.loss)
     assert torch.equal(out.dlogits, ref_out.dlogits)
+
+
+@pytest.mark.parametrize("T,E,k,gate,routed", [
+    (4096 + 33, 128, 8, 0, True),     # ALU loss kernel with a summed D (no tensor-core image)
+    (4096 + 33, 128, 8, 0, False),
+    (2048, 64, 4, 1, True),
+    (999, 33, 3, 0, True),            # generic kernels
+])
+def test_backward_half_with_a_summed_matrix(dl, T, E, k, gate, routed):
+    """Global-DO (Sec. 3.1.4, Eq. global_do) through the halves: the forward
+    half's local D plus another rank's, d_scale = 1/2, m = the local T; the
+    loss and gradient as the oracle computes them with that matrix, plus the
+    routing gradient when asked."""
+    z = workloads.random_logits(T, E, seed=T + 5)
+    z_other = workloads.random_logits(T + 100, E, seed=T + 6)
+    out, route = dl.routed_forward(z.cuda(), k, gate, with_routing=routed)
+    zl = z[0].numpy()
+    f = oracle.select(zl, k)
+    D_sum = oracle.hamming(f) + oracle.hamming(oracle.select(z_other[0].numpy(), k))
+    Dg = torch.from_numpy(D_sum.astype(np.int32))[None].cuda()
+    grad = torch.randn(1, T, k, generator=torch.Generator().manual_seed(1)).cuda()
+    dl.routed_backward(z.cuda(), route.expert_ids if routed else None, grad if routed else None,
+                       k, gate, 0.75, out=out, D=Dg, d_scale=0.5)
+    torch.cuda.synchronize()
+    assert dl.device_status(out.workspace) == 0
+    want_loss = oracle.loss(D_sum, oracle.direction(zl, f, gate), T, k, 0.5)
+    assert abs(float(out.loss[0]) - want_loss) <= 1e-5 * abs(want_loss)
+    g_do = 0.75 * oracle.gate_backward(zl, oracle.dloss_dp(D_sum, f, T, k, d_scale=0.5), gate)
+    tol = 1e-4 * np.abs(g_do).max()
+    want = g_do
+    if routed:
+        ids, _ = oracle.route(zl, k, gate)
+        gl = grad[0].cpu().numpy()
+        want = want + oracle.route_backward(zl, ids, gl.astype(np.float64), gate)
+        tol = tol + route_bound(zl, ids, gl, gate)
+    assert (np.abs(out.dlogits[0].double().cpu().numpy() - want) <= tol).all()
+
+
+def test_global_do_binding_at_one_rank_is_the_local_step(dl):
+    """global_forward_backward through the halves with no process group:
+    d_scale = 1, the tensor-core path, bit for bit do_forward_backward."""
+    w = workloads.get("c3", T=8192)
+    z = workloads.logits(w).cuda()
+    loss, dz, D, counts = dl.global_forward_backward(z, w.k, w.gate, grad_scale=2.0)
+    ref = dl.forward_backward(z, w.k, w.gate, grad_scale=2.0)
+    torch.cuda.synchronize()
+    assert torch.equal(D, ref.D) and torch.equal(counts, ref.counts)
+    assert torch.equal(loss, ref.loss) and torch.equal(dz, ref.dlogits)
