@@ -98,6 +98,13 @@ do_status do_pairwise_hamming(const uint32_t *bits, int64_t T, int32_t E, int32_
 do_status do_pairwise_hamming_accumulate(const uint32_t *bits, int64_t T, int32_t E, int32_t L,
                                          int32_t *D, void *stream);
 
+/* D_sum += D for [L][E][E] int32 Hamming matrices (device): the matrices of
+ * the micro-batches of an accumulation window add up before the loss
+ * (Eq. global_do).  Integer, exact while each sum stays within int32 (the
+ * window's tokens below 2^31).  Asynchronous on `stream`. */
+do_status do_accumulate_distances(const int32_t *D, int32_t E, int32_t L, int32_t *D_sum,
+                                  void *stream);
+
 /* Step 3 (Sec. 3.1.3, Eq. do_loss; Sec. 3.1.4, Eq. global_do):
  *   L_DO = 1/(T^2 k) sum_i sum_j G_ij C_ij,  C_ij = sum_t p_it (f_it - f_jt),
  * with G = d_scale * D held constant (detached) and p the dense router

@@ -157,6 +157,15 @@ do_status do_pairwise_hamming_accumulate(const uint32_t *bits, int64_t T, int32_
     return from_cuda(dol::launch_hamming_accumulate(bits, p, D, nullptr, (cudaStream_t)stream));
 }
 
+do_status do_accumulate_distances(const int32_t *D, int32_t E, int32_t L, int32_t *D_sum,
+                                  void *stream) {
+    NvtxRange nvtx("do_accumulate_distances");
+    if (!D || !D_sum || E < 1 || L < 1 || !aligned(D, 4) || !aligned(D_sum, 4))
+        return DO_ERR_INVALID_ARG;
+    if (E > 1024 || L > 65535) return DO_ERR_UNSUPPORTED;
+    return from_cuda(dol::launch_add_distances(D, D_sum, (int64_t)L * E * E, (cudaStream_t)stream));
+}
+
 do_status do_loss_fwd_bwd(const float *logits, const uint32_t *bits, const int32_t *D, int64_t T,
                           int32_t E, int32_t k, int32_t L, int32_t gate, float d_scale,
                           float grad_scale, float *loss, int64_t *origin_do, float *dlogits,

@@ -138,4 +138,35 @@ cudaError_t launch_hamming(const uint32_t *bits, const Problem &p, int *D, cudaS
     return launch_hamming_accumulate(bits, p, D, nullptr, s);
 }
 
+// D_sum += D over n int32 entries (the Hamming matrices of the micro-batches
+// of a window add up, Eq. global_do); a grid-stride loop of 16-byte rows
+// where both are aligned.
+__global__ void __launch_bounds__(256)
+add_distances_kernel(const int *__restrict__ D, int *__restrict__ D_sum, int64_t n, int vec) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (vec) {
+        const int4 *a = reinterpret_cast<const int4 *>(D);
+        int4 *b = reinterpret_cast<int4 *>(D_sum);
+        for (int64_t i = t; i < n / 4; i += stride) {
+            const int4 x = __ldg(a + i);
+            int4 y = b[i];
+            y.x += x.x; y.y += x.y; y.z += x.z; y.w += x.w;
+            b[i] = y;
+        }
+        for (int64_t i = (n / 4) * 4 + t; i < n; i += stride) D_sum[i] += __ldg(D + i);
+    } else {
+        for (int64_t i = t; i < n; i += stride) D_sum[i] += __ldg(D + i);
+    }
+}
+
+cudaError_t launch_add_distances(const int *D, int *D_sum, int64_t n, cudaStream_t s) {
+    const int vec = (reinterpret_cast<uintptr_t>(D) % 16 == 0 &&
+                     reinterpret_cast<uintptr_t>(D_sum) % 16 == 0) ? 1 : 0;
+    const int64_t want = ((vec ? (n + 3) / 4 : n) + 255) / 256;
+    const int blocks = (int)(want < 1 ? 1 : (want > 1024 ? 1024 : want));
+    add_distances_kernel<<<blocks, 256, 0, s>>>(D, D_sum, n, vec);
+    return cudaGetLastError();
+}
+
 }  // namespace dol

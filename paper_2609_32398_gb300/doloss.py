@@ -47,6 +47,7 @@ EXPORTS = {
     "do_routing_workspace_size": (["i64", "i32", "i32", "i32"], "sz"),
     "do_route_backward": (["p", "p", "p", "i64", "i32", "i32", "i32", "i32", "i32", "p", "p", "p"],
                           "i32"),
+    "do_accumulate_distances": (["p", "i32", "i32", "p", "p"], "i32"),
     "do_routed_forward": (["p", "i64", "i32", "i32", "i32", "i32", "p", "p", "p", "p", "p", "p", "p",
                            "p", "p", "p", "sz", "p"], "i32"),
     "do_routed_backward": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "f32", "p", "p", "p", "p",
@@ -573,7 +574,7 @@ def global_forward_backward(logits, k, gate=GATE_SIGMOID_NORM, grad_scale=1.0, g
 def window_forward_backward(logits_list, k, gate=GATE_SIGMOID_NORM, grad_scale=1.0, group=None):
     """Global-DO over a gradient-accumulation window (Sec. 3.1.4, Eq. global_do;
     App. batch ablation): the Hamming matrices of the window's micro-batches
-    are summed (do_pairwise_hamming_accumulate), then summed over the ranks of
+    (each from its forward half) are summed, then summed over the ranks of
     `group`, and every micro-batch's loss and gradient use that matrix with
     d_scale = 1 / (ranks x micro-batches) and m = its own token count.
     logits_list: the window's micro-batches, each [L,T,E] or [T,E] on the GPU.
@@ -583,23 +584,21 @@ def window_forward_backward(logits_list, k, gate=GATE_SIGMOID_NORM, grad_scale=1
         raise ValueError("an empty window")
     L, _, E = zs[0].shape
     D = torch.zeros(L, E, E, dtype=torch.int32, device=zs[0].device)
-    sigs = []
+    outs = []
     for z in zs:
         if z.shape[0] != L or z.shape[2] != E:
             raise ValueError("the window's micro-batches must share L and E")
-        bits, _ = signatures(z, k)
-        _check("do_pairwise_hamming_accumulate", lib().do_pairwise_hamming_accumulate(
-            bits.data_ptr(), z.shape[1], E, L, D.data_ptr(), _stream(z)))
-        sigs.append(bits)
+        # the forward half of each micro-batch (its own buffers: the backward
+        # half reads the selection it leaves), its matrix added to the window's
+        out, _ = routed_forward(z, k, gate, with_routing=False)
+        _check("do_accumulate_distances", lib().do_accumulate_distances(
+            out.D.data_ptr(), E, L, D.data_ptr(), _stream(z)))
+        outs.append(out)
     D, d_rank = all_reduce_distances(D, group)
     d_scale = d_rank / len(zs)
-    losses, grads = [], []
-    for z, bits in zip(zs, sigs):
-        loss, _, dz = loss_fwd_bwd(z, bits, D, k, gate, d_scale=d_scale, grad_scale=grad_scale,
-                                   with_origin=False)
-        losses.append(loss)
-        grads.append(dz)
-    return losses, grads, D
+    for z, out in zip(zs, outs):
+        routed_backward(z, None, None, k, gate, grad_scale, out=out, D=D, d_scale=d_scale)
+    return [o.loss for o in outs], [o.dlogits for o in outs], D
 
 
 class _DOLossFunction(torch.autograd.Function):

@@ -203,3 +203,14 @@ def test_routed_halves_validate_on_the_host(dl):
     # steps 1-2 alone: routing outputs absent, but then no dispatch arrays either
     assert f(fake, 64, 8, 2, 1, 0, fake, fake, fake, None, None, None, fake, None, None, fake, big,
              None) == INV
+
+
+def test_accumulate_distances_validates_on_the_host(dl):
+    lib = dl.lib()
+    fake = ctypes.c_void_p(0x10000)
+    odd = ctypes.c_void_p(0x10002)
+    assert lib.do_accumulate_distances(None, 8, 1, fake, None) == 1
+    assert lib.do_accumulate_distances(fake, 8, 1, None, None) == 1
+    assert lib.do_accumulate_distances(fake, 0, 1, fake, None) == 1
+    assert lib.do_accumulate_distances(odd, 8, 1, fake, None) == 1
+    assert lib.do_accumulate_distances(fake, 2048, 1, fake, None) == 2

@@ -111,3 +111,21 @@ def test_accumulation_window_matches_oracle():
         assert abs(float(loss[0]) - want) <= 1e-5 * abs(want)
         g = oracle.gate_backward(zl, oracle.dloss_dp(D_ref, f, T, k, d_scale=1.0 / 3))
         assert np.abs(dz[0].double().cpu().numpy() - g).max() <= 1e-4 * np.abs(g).max()
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("E,L,offset", [(128, 1, 0), (33, 3, 1), (256, 2, 0)])
+def test_accumulate_distances_is_the_integer_sum(E, L, offset):
+    """do_accumulate_distances adds [L,E,E] int32 matrices exactly, on the
+    16-byte path and (one-element offset) the scalar one."""
+    import paper_2609_32398_gb300.doloss as dl
+
+    g = torch.Generator().manual_seed(E + L)
+    a = torch.randint(0, 1 << 20, (L * E * E + offset,), generator=g, dtype=torch.int32).cuda()
+    b = torch.randint(0, 1 << 20, (L * E * E + offset,), generator=g, dtype=torch.int32).cuda()
+    want = (a.long() + b.long())[offset:]
+    st = dl.lib().do_accumulate_distances(a[offset:].data_ptr(), E, L, b[offset:].data_ptr(),
+                                          torch.cuda.current_stream().cuda_stream)
+    assert st == 0
+    torch.cuda.synchronize()
+    assert torch.equal(b[offset:].long(), want)
