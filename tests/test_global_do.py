@@ -129,3 +129,58 @@ def test_accumulate_distances_is_the_integer_sum(E, L, offset):
     assert st == 0
     torch.cuda.synchronize()
     assert torch.equal(b[offset:].long(), want)
+
+
+def _gpu_rank_main(rank, world, port, out):
+    os.environ.update({"MASTER_ADDR": "127.0.0.1", "MASTER_PORT": str(port), "RANK": str(rank),
+                       "WORLD_SIZE": str(world)})
+    sys.path.insert(0, ROOT)
+    import torch.distributed as dist
+
+    from paper_2609_32398_gb300 import doloss, workloads
+
+    torch.cuda.set_device(0)
+    dist.init_process_group("gloo")
+    w = workloads.get("c3", T=8192)
+    z = workloads.logits(w)[0]
+    shard = z[rank * 4096:(rank + 1) * 4096].contiguous().cuda()
+    loss, dz, D, counts = doloss.global_forward_backward(shard, w.k, w.gate, grad_scale=1.0)
+    torch.cuda.synchronize()
+    out[rank] = (float(loss[0]), dz[0].cpu().numpy(), D[0].cpu().numpy(), counts[0].cpu().numpy())
+    dist.destroy_process_group()
+
+
+@pytest.mark.gpu
+def test_two_gloo_ranks_on_the_gpu_path():
+    """Global-DO through the GPU halves with a real process group: two ranks
+    (processes on one GPU; the only exchange is gloo's host all-reduce of D,
+    none of the kernels waits on another rank) each hold half of the c3
+    tokens.  The summed D is the oracle's matrix of all tokens, and each
+    rank's loss and gradient are the oracle's for its shard with d_scale = 1/2
+    (the ALU loss kernel)."""
+    import oracle
+    from paper_2609_32398_gb300 import workloads
+
+    ctx = mp.get_context("spawn")
+    manager = ctx.Manager()
+    out = manager.dict()
+    port = _free_port()
+    procs = [ctx.Process(target=_gpu_rank_main, args=(r, 2, port, out)) for r in range(2)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(timeout=300)
+    assert all(p.exitcode == 0 for p in procs)
+    w = workloads.get("c3", T=8192)
+    z = workloads.logits(w)[0].numpy()
+    D_all = oracle.hamming(oracle.select(z, w.k))
+    for r in range(2):
+        loss, dz, D, counts = out[r]
+        assert np.array_equal(D, D_all)
+        shard = z[r * 4096:(r + 1) * 4096]
+        f = oracle.select(shard, w.k)
+        assert np.array_equal(counts, oracle.counts(f))
+        want = oracle.loss(D_all, oracle.direction(shard, f, w.gate), 4096, w.k, 0.5)
+        assert abs(loss - want) <= 1e-5 * abs(want)
+        g = oracle.gate_backward(shard, oracle.dloss_dp(D_all, f, 4096, w.k, d_scale=0.5), w.gate)
+        assert np.abs(dz - g).max() <= 1e-4 * np.abs(g).max()
