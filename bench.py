@@ -22,6 +22,7 @@ import argparse
 import hashlib
 import json
 import os
+import platform
 import re
 import statistics
 import subprocess
@@ -87,6 +88,21 @@ def router_bytes(T, E, H, L=1):
     signature, Hamming-matrix and count traffic of the DO-loss path."""
     W = (T + 31) // 32
     return L * (2 * T * H + 2 * E * H + 12 * T * E + 8 * E * W + 8 * E * E + 4 * E)
+
+
+def host_cpu():
+    """The host's CPU model and logical core count (context for the oracle
+    baseline, which uses one core)."""
+    model = None
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.split(":")[0].strip() in ("Model name", "BIOS Model name") and ":" in line:
+                model = line.split(":", 1)[1].strip()
+                break
+    except Exception:
+        pass
+    return {"model": model or platform.machine(), "logical_cores": os.cpu_count()}
 
 
 def measured_peaks():
@@ -277,7 +293,8 @@ def run_reference(args, rank, world):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": config_dict(w),
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc,
+                         "host": host_cpu()},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -655,7 +672,8 @@ def run_ours(args, rank, world, local):
         rate, ntok, spent, runs = oracle_throughput(zc, k, w.gate, budget_s=10.0)
         cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
                "sample": f"{runs} oracle run(s) over all {T} tokens of the same workload "
-                         f"({spent:.1f} s, single-threaded C, double precision)"}
+                         f"({spent:.1f} s, single-threaded C, double precision)",
+               "host": host_cpu()}
 
     if rank == 0:
         line = {

@@ -184,3 +184,20 @@ def test_two_gloo_ranks_on_the_gpu_path():
         assert abs(loss - want) <= 1e-5 * abs(want)
         g = oracle.gate_backward(shard, oracle.dloss_dp(D_all, f, 4096, w.k, d_scale=0.5), w.gate)
         assert np.abs(dz - g).max() <= 1e-4 * np.abs(g).max()
+
+
+@pytest.mark.gpu
+def test_window_of_one_micro_batch_is_the_local_step():
+    """A window of one micro-batch on one rank has d_scale = 1: the backward
+    half takes the tensor-core kernel and returns do_forward_backward's loss
+    and dlogits bit for bit."""
+    import paper_2609_32398_gb300.doloss as dl
+    from paper_2609_32398_gb300 import workloads
+
+    w = workloads.get("c3", T=4096 + 17)
+    z = workloads.logits(w).cuda()
+    losses, grads, D = dl.window_forward_backward([z], w.k, w.gate, grad_scale=1.5)
+    ref = dl.forward_backward(z, w.k, w.gate, grad_scale=1.5)
+    torch.cuda.synchronize()
+    assert torch.equal(D, ref.D)
+    assert torch.equal(losses[0], ref.loss) and torch.equal(grads[0], ref.dlogits)
