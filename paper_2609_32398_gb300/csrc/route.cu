@@ -116,6 +116,21 @@ route_scatter_kernel(const uint32_t *__restrict__ bits, const int *__restrict__ 
     const int Tk = T * k;
     const int i0 = (int)(32 * w0) * k, i1 = (int)min64(T, 32 * (w0 + nw)) * k;
     const int *il = ids + (size_t)layer * Tk;
+    // this thread's experts' totals and chunk bases (at most four consecutive
+    // experts per thread, E <= 1024), loaded with everything else up front so
+    // that the kernel waits for one round trip of loads, not three
+    const int per = (E + kScatterThreads - 1) / kScatterThreads;
+    int tot_v[4], cb_v[4];
+    {
+        const int *tl = totals + (size_t)layer * E;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int e = tid * per + j;
+            const bool on = j < per && e < E;
+            tot_v[j] = on ? __ldg(tl + e) : 0;
+            cb_v[j] = on ? __ldg(chunk_base + ((size_t)layer * E + e) * nchunks + c) : 0;
+        }
+    }
     // the first batch of this thread's expert ids: loaded before the barriers
     // below, so that its latency overlaps the shared-memory set-up
     int ev[kBatch];
@@ -144,15 +159,11 @@ route_scatter_kernel(const uint32_t *__restrict__ bits, const int *__restrict__ 
     {
         __shared__ int s_wsum[kScatterThreads / 32];
         const int lane = tid & 31, wp = tid >> 5;
-        const int per = (E + kScatterThreads - 1) / kScatterThreads;
-        const int *tl = totals + (size_t)layer * E;
         int loc[4], sum = 0;
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-            const int e = tid * per + j;
-            const int v = (j < per && e < E) ? __ldg(tl + e) : 0;
             loc[j] = sum;
-            sum += v;
+            sum += tot_v[j];
         }
         int x = sum;
 #pragma unroll
@@ -173,7 +184,7 @@ route_scatter_kernel(const uint32_t *__restrict__ bits, const int *__restrict__ 
         for (int j = 0; j < 4; ++j) {
             const int e = tid * per + j;
             if (j < per && e < E) {
-                s_cb[e] = excl + loc[j] + chunk_base[((size_t)layer * E + e) * nchunks + c];
+                s_cb[e] = excl + loc[j] + cb_v[j];
                 if (offsets && c == 0) offsets[(size_t)layer * (E + 1) + e] = excl + loc[j];
             }
         }
