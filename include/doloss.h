@@ -10,10 +10,13 @@
  *   3. the surrogate loss and its gradient to the router logits
  *                                                       (Sec. 3.1.3, Eq. do_loss)
  *   4. Eq. origin_do, the sum of squared distances, as a diagnostic.
- * and around them: the router's outputs (do_routing), the router's linear map
- * fused with step 1 and its backward (do_router_forward_backward,
- * do_router_backward), and the consumers of the counts (do_maxvio,
- * do_rem_allocate).
+ * and around them: the router's outputs (do_routing) and their backward
+ * (do_route_backward), the routed step in the forward and backward halves of
+ * a training step (do_routed_forward, do_routed_backward; also the per-rank
+ * step of Global-DO, with do_accumulate_distances for accumulation windows),
+ * the router's linear map fused with step 1 and its backward
+ * (do_router_forward_backward, do_router_backward), and the consumers of the
+ * counts (do_maxvio, do_rem_allocate).
  *
  * Notation: E experts (the paper's n), k selected per token (K), T tokens in
  * the signature window (m), L independent problems batched in one call (for
@@ -25,15 +28,17 @@
  *    and do_rem_allocate, a host function.  The library allocates nothing and
  *    keeps no state between calls, with two stated exceptions:
  *    do_forward_backward_static (a fixed scratch array per device) and
- *    do_router_backward (a cuBLAS handle per device).
+ *    do_router_backward (a cuBLAS handle per device).  do_routed_backward
+ *    reads what do_routed_forward left in the caller's workspace.
  *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default
  *    stream).  Calls are asynchronous on it, except do_device_status and
  *    do_forward_backward_host, which synchronize it.
  *  - Arguments are validated before anything is launched; a rejected call
  *    returns DO_ERR_INVALID_ARG or DO_ERR_UNSUPPORTED and touches no memory.
  *    A failed launch returns DO_ERR_CUDA.  Conditions only the device can see
- *    (a Hamming row sum that does not fit int32, a device wait that ran out)
- *    are recorded in the workspace and reported by do_device_status.
+ *    (a Hamming row sum that does not fit int32, a device wait that ran out,
+ *    an expert id out of range given to do_routed_backward) are recorded in
+ *    the workspace and reported by do_device_status.
  *  - Layouts are dense and row-major:
  *      logits, dlogits  [L][T][E] fp32 (token-major: one row per token)
  *      bits             [L][E][W] uint32; bit (t mod 32) of word t/32 of row i
@@ -50,7 +55,8 @@
  *    the vectorised kernels); uint32/int32 arrays 4-byte, int64 8-byte.
  *  - Results are deterministic: bits, counts, D and origin_do are exact
  *    integers; loss and dlogits are bitwise reproducible run to run (fixed
- *    reduction order, no floating-point atomics).
+ *    reduction order; the one floating-point atomic, do_route_backward's
+ *    accumulate mode, adds once to each entry).
  */
 #ifndef DOLOSS_H
 #define DOLOSS_H
