@@ -154,3 +154,28 @@ def test_route_backward_equal_chosen_logits_closed_form(c, gate):
     want = (g - g.mean(1, keepdims=True)) / k * factor
     np.testing.assert_allclose(np.take_along_axis(dz, ids.astype(np.int64), axis=1), want,
                                rtol=1e-12, atol=0)
+
+
+def _value(v):
+    if v.lstrip("-") == "sig(-1)":
+        x = 1.0 / (1.0 + np.e)
+        return -x if v.startswith("-") else x
+    return float(Fraction(v))
+
+
+def test_route_backward_worked_example():
+    """The combine weights' gradient on the hand-worked tokens of the routing
+    example (tests/golden/route_backward_worked_n4_k2.json)."""
+    g = json.load(open(os.path.join(GOLDEN, "route_backward_worked_n4_k2.json")))
+    z = np.array([[_sym(v) for v in row] for row in g["logits_symbolic"]], np.float32)
+    ids = np.array(g["expert_ids"], np.int32)
+    grad = np.array(g["grad_combine"], np.float64)
+    for gate, key in ((oracle.GATE_SIGMOID_NORM, "dlogits_sigmoid_norm"),
+                      (oracle.GATE_SOFTMAX, "dlogits_softmax")):
+        got_ids, _ = oracle.route(z, g["K"], gate)
+        assert got_ids.tolist() == g["expert_ids"]
+        want = np.array([[_value(v) for v in row] for row in g[key]])
+        dz = oracle.route_backward(z, ids, grad, gate)
+        # the logits are fp32 roundings of ln 2 and ln 3: agreement to their rounding
+        np.testing.assert_allclose(dz, want, rtol=0, atol=2e-7)
+        assert (dz[want == 0] == 0).all()

@@ -216,3 +216,30 @@ def test_autograd_route_with_the_do_loss(dl, gate):
     tol = 1e-4 * np.abs(want_do).max() + bound(zl, ids_ref, u.cpu().numpy(), gate)
     got = z.grad.double().cpu().numpy()
     assert (np.abs(got - (want_route + want_do)) <= tol).all()
+
+
+def test_route_backward_worked_example_on_the_gpu(dl):
+    """The hand-worked tokens of tests/golden/route_backward_worked_n4_k2.json
+    through do_route_backward (E = 4: the gather kernel's unaligned-width
+    path), both gates."""
+    import json
+    import os
+    from fractions import Fraction
+
+    g = json.load(open(os.path.join(os.path.dirname(__file__), "golden",
+                                    "route_backward_worked_n4_k2.json")))
+    sym = {"0": 0.0, "1": 1.0, "ln2": np.log(2.0), "-ln2": -np.log(2.0), "ln3": np.log(3.0),
+           "-ln3": -np.log(3.0)}
+    z = torch.tensor([[sym[v] for v in row] for row in g["logits_symbolic"]], dtype=torch.float32)
+    ids = torch.tensor(g["expert_ids"], dtype=torch.int32)
+    grad = torch.tensor(g["grad_combine"], dtype=torch.float32)
+
+    def value(v):
+        if v.lstrip("-") == "sig(-1)":
+            x = 1.0 / (1.0 + np.e)
+            return -x if v.startswith("-") else x
+        return float(Fraction(v))
+    for gate, key in ((0, "dlogits_sigmoid_norm"), (1, "dlogits_softmax")):
+        dz = dl.route_backward(z.cuda(), ids.cuda(), grad.cuda(), gate)
+        want = np.array([[value(v) for v in row] for row in g[key]])
+        np.testing.assert_allclose(dz.double().cpu().numpy()[0], want, rtol=0, atol=1e-6)
