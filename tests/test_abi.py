@@ -214,3 +214,38 @@ def test_accumulate_distances_validates_on_the_host(dl):
     assert lib.do_accumulate_distances(fake, 0, 1, fake, None) == 1
     assert lib.do_accumulate_distances(odd, 8, 1, fake, None) == 1
     assert lib.do_accumulate_distances(fake, 2048, 1, fake, None) == 2
+
+
+def _ctype_code(decl):
+    """The binding's argument code of one C parameter or return type."""
+    d = " ".join(decl.replace("const ", "").split())
+    if "*" in d:
+        return "str" if d.startswith("char") else "p"
+    base = d.split()[0]
+    return {"int64_t": "i64", "int32_t": "i32", "float": "f32", "size_t": "sz", "do_status": "i32",
+            "double": "f64"}[base]
+
+
+def declared_signatures():
+    text = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    out = {}
+    for ret, name, params in re.findall(r"([A-Za-z_][\w \*]*?)\s*\b(do_[a-z_0-9]+)\s*\(([^)]*)\)\s*;",
+                                        text):
+        ret = ret.split()[-1] if "*" not in ret else ret
+        args = [p.strip() for p in params.split(",") if p.strip() and p.strip() != "void"]
+        # drop the parameter name: what precedes the last identifier is the type
+        types = [re.sub(r"\b\w+\s*$", "", a).strip() or a for a in args]
+        out[name] = ([_ctype_code(t) for t in types], _ctype_code(ret))
+    return out
+
+
+def test_binding_signatures_match_the_header(dl):
+    """Every declared function's parameter kinds (pointer, int32, int64, float,
+    size_t) and result kind, read from include/doloss.h, are those the ctypes
+    binding declares, so that a changed signature cannot go unnoticed."""
+    sigs = declared_signatures()
+    assert set(sigs) == set(declared_functions())
+    for name, (args, res) in sigs.items():
+        want_args, want_res = dl.EXPORTS[name]
+        assert args == want_args, (name, args, want_args)
+        assert res == want_res, (name, res, want_res)
