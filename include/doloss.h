@@ -104,6 +104,16 @@ do_status do_pairwise_hamming(const uint32_t *bits, int64_t T, int32_t E, int32_
 do_status do_pairwise_hamming_accumulate(const uint32_t *bits, int64_t T, int32_t E, int32_t L,
                                          int32_t *D, void *stream);
 
+/* The variance of the E (E - 1) off-diagonal distances of each problem's
+ * local Hamming matrix, the dispersion that Eq. origin_do measures (App. C.1):
+ * with Eq. zero_sum their mean is 2 T k (E - k) / (E (E - 1)), so
+ *   var[l] = origin_do[l] / (E (E - 1)) - mean^2    (fp64),
+ * without reading D.  origin_do [L] int64 as the fused calls write it (a
+ * window of T tokens with k experts each; not a matrix summed over ranks);
+ * var [L] fp64.  Needs E >= 2.  Asynchronous on `stream`. */
+do_status do_offdiag_variance(const int64_t *origin_do, int64_t T, int32_t E, int32_t k, int32_t L,
+                              double *var, void *stream);
+
 /* D_sum += D for [L][E][E] int32 Hamming matrices (device): the matrices of
  * the micro-batches of an accumulation window add up before the loss
  * (Eq. global_do).  Integer, exact while each sum stays within int32 (the
@@ -135,9 +145,9 @@ do_status do_loss_fwd_bwd(const float *logits, const uint32_t *bits, const int32
  * counts, D, loss, origin_do (may be NULL) and dlogits (may be NULL) out.
  * With E = 128, the sigmoid-normalised gate, k in {1, 2, 4, 8}, T <= 66052
  * and dlogits given, the gradient pass computes V = F D' on the tensor cores
- * (F the one-hot selections, D' = D with -R on the diagonal); elsewhere, or
- * with the environment variable DOLOSS_LOSS_KERNEL=alu, it gathers rows of D'
- * on the ALU.  The two agree within the stated tolerances. */
+ * (F the one-hot selections, D' = D with -R on the diagonal); elsewhere it
+ * gathers rows of D' on the ALU (as do_loss_fwd_bwd always does).  The two
+ * agree within the stated tolerances. */
 do_status do_forward_backward(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
                               int32_t gate, float grad_scale, uint32_t *bits, int32_t *counts,
                               int32_t *D, float *loss, int64_t *origin_do, float *dlogits,
@@ -361,11 +371,13 @@ do_status do_forward_backward_host_async(const float *h_logits, int64_t T, int32
  *  - Sizes whose do_workspace_size exceeds DO_STATIC_SCRATCH_BYTES are
  *    rejected with DO_ERR_WORKSPACE before anything is launched (for
  *    E = 128, k = 8, L = 1 that is T above about 0.97 million tokens).
- *  - Unlike the other entry points it keeps state: the first call on a device
- *    (with that device current) looks up the array's address, zero-fills the
- *    array and synchronizes the device; make that first call before any
- *    stream capture begins.  Every call then clears the parts that must start
- *    at zero with cudaMemsetAsync on `stream`.
+ *  - Unlike the other entry points it keeps state: the first call in a CUDA
+ *    context (with its device current) looks up the array's device address
+ *    and caches it for that context (a context created later, e.g. after
+ *    cudaDeviceReset, looks it up again); make that first call before any
+ *    stream capture begins.  Every call clears the parts that must start at
+ *    zero with cudaMemsetAsync on `stream`; the array keeps the rest of the
+ *    last call's contents.
  *  - status_flags (device int32, may be NULL) receives the device status
  *    word of this call, copied on `stream`: bit 0 = a Hamming row sum did
  *    not fit int32, bit 1 = a bounded device wait ran out.

@@ -4,7 +4,6 @@
 
 #include <climits>
 #include <cstdint>
-#include <cstdlib>
 #include <cstring>
 
 #include <nvtx3/nvToolsExt.h>
@@ -34,14 +33,6 @@ do_status check_sizes(int64_t T, int32_t E, int32_t k, int32_t L, Problem *p) {
     p->L = L;
     p->W = (T + 31) / 32;
     return DO_OK;
-}
-
-// The fused path takes the tensor-core loss kernel (one-hot selections times
-// D' on tcgen05) wherever it applies; DOLOSS_LOSS_KERNEL=alu selects the ALU
-// kernel (a shared-memory gather of D rows) instead.
-bool alu_loss_requested() {
-    const char *v = std::getenv("DOLOSS_LOSS_KERNEL");
-    return v && std::strcmp(v, "alu") == 0;
 }
 
 do_status from_cuda(cudaError_t e) { return e == cudaSuccess ? DO_OK : DO_ERR_CUDA; }
@@ -157,6 +148,18 @@ do_status do_pairwise_hamming_accumulate(const uint32_t *bits, int64_t T, int32_
     return from_cuda(dol::launch_hamming_accumulate(bits, p, D, nullptr, (cudaStream_t)stream));
 }
 
+do_status do_offdiag_variance(const int64_t *origin_do, int64_t T, int32_t E, int32_t k, int32_t L,
+                              double *var, void *stream) {
+    NvtxRange nvtx("do_offdiag_variance");
+    Problem p;
+    do_status st = check_sizes(T, E, k, L, &p);
+    if (st != DO_OK) return st;
+    if (E < 2 || !origin_do || !var || !aligned(origin_do, 8) || !aligned(var, 8))
+        return DO_ERR_INVALID_ARG;
+    return from_cuda(dol::launch_offdiag_variance(reinterpret_cast<const long long *>(origin_do), p,
+                                                  var, (cudaStream_t)stream));
+}
+
 do_status do_accumulate_distances(const int32_t *D, int32_t E, int32_t L, int32_t *D_sum,
                                   void *stream) {
     NvtxRange nvtx("do_accumulate_distances");
@@ -253,8 +256,7 @@ do_status forward_backward_impl(const float *logits, int64_t T, int32_t E, int32
         int *status = reinterpret_cast<int *>(ws);
         // D <= T here (one window of tokens): the two-piece fp16 split of the
         // tensor-core path is exact when R < 2^23 (checked by loss_mma_supported)
-        const bool mma = !alu_loss_requested() &&
-                         dol::loss_mma_supported(p, gate, logits, D, dlogits);
+        const bool mma = dol::loss_mma_supported(p, gate, logits, D, dlogits);
         unsigned char *bimg = mma ? reinterpret_cast<unsigned char *>(ws + w.bimg) : nullptr;
         cudaError_t e =
             rin ? dol::launch_router_signatures(rin->X, rin->Wr, rin->H, const_cast<float *>(logits),
@@ -352,7 +354,7 @@ bool split_fast(const Problem &p, const float *logits, const uint32_t *bits, con
 // Whether the forward half writes the fp16 image of D' for the tensor-core
 // loss kernel (dlogits is not known there: the logits' alignment stands in).
 bool split_mma(const Problem &p, int gate, const float *logits, const int *D) {
-    return !alu_loss_requested() && dol::loss_mma_supported(p, gate, logits, D, logits);
+    return dol::loss_mma_supported(p, gate, logits, D, logits);
 }
 
 do_status do_routed_forward(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,

@@ -21,13 +21,6 @@ constexpr int kRedWarps = 32;
 constexpr int kRedThreads = kRedWarps * 32;
 static_assert(kMaxSigCtas <= 8 * kRedWarps, "a warp adds at most eight partials");
 
-__device__ __forceinline__ void put_pieces(unsigned char *img, int n, int k, bool diag, int v) {
-    int h, l;
-    dprime_pieces(diag, v, &h, &l);
-    *reinterpret_cast<__half *>(img + sw128_k16_offset(n, k, 256)) = __int2half_rn(h);
-    *reinterpret_cast<__half *>(img + sw128_k16_offset(128 + n, k, 256)) = __int2half_rn(l);
-}
-
 template <int E>
 __global__ void __launch_bounds__(kRedThreads)
 cooc_reduce_kernel(const uint32_t *__restrict__ partials, int P1, const int *__restrict__ n_acc,
@@ -78,14 +71,14 @@ cooc_reduce_kernel(const uint32_t *__restrict__ partials, int P1, const int *__r
             Dl[a * E + a] = 0;
             counts[(size_t)layer * E + a] = (int)c;
             // R_a = (E - 2k) n_a + T k (every row of the co-occurrence sums to k n_a)
-            if (img) put_pieces(img, a, a, true, (int)(r_base + (long long)r_mult * (long long)c));
+            if (img) put_dprime(img, a, a, true, (int)(r_base + (long long)r_mult * (long long)c));
         } else {
             const int d = s_n[a] + s_n[b] - 2 * (int)c;
             Dl[a * E + b] = d;
             Dl[b * E + a] = d;
             if (img) {
-                put_pieces(img, a, b, false, d);
-                put_pieces(img, b, a, false, d);
+                put_dprime(img, a, b, false, d);
+                put_dprime(img, b, a, false, d);
             }
             sq = 2 * (long long)d * (long long)d;
         }

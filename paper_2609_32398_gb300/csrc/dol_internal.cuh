@@ -2,6 +2,7 @@
 // Nothing here is part of the public interface (include/doloss.h is).
 #pragma once
 
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 #include <stdint.h>
@@ -97,6 +98,10 @@ cudaError_t launch_add_distances(const int *D, int *D_sum, int64_t n, cudaStream
 cudaError_t launch_hamming_accumulate(const uint32_t *bits, const Problem &p, int *D, int *counts,
                                       cudaStream_t s);
 cudaError_t launch_origin_do(const int *D, const Problem &p, long long *origin_do, cudaStream_t s);
+// var [L] (fp64) = the variance of the off-diagonal entries of each problem's
+// local Hamming matrix from its origin_do (App. C.1).
+cudaError_t launch_offdiag_variance(const long long *origin_do, const Problem &p, double *var,
+                                    cudaStream_t s);
 cudaError_t launch_loss(const float *logits, const uint32_t *bits, const int *D,
                         const Problem &p, int gate, float d_scale, float grad_scale,
                         float *loss, long long *origin_do, float *dlogits, void *workspace,
@@ -195,6 +200,15 @@ __host__ __device__ __forceinline__ void dprime_pieces(bool diag, int v, int *hi
     }
 }
 
+// Writes the two fp16 pieces of D'_{n,k} (dprime_pieces) into the image at
+// row n (hi) and row 128 + n (lo), column k.
+__device__ __forceinline__ void put_dprime(unsigned char *img, int n, int k, bool diag, int v) {
+    int h, l;
+    dprime_pieces(diag, v, &h, &l);
+    *reinterpret_cast<__half *>(img + sw128_k16_offset(n, k, 256)) = __int2half_rn(h);
+    *reinterpret_cast<__half *>(img + sw128_k16_offset(128 + n, k, 256)) = __int2half_rn(l);
+}
+
 int sig_fast_ctas_per_problem(const Problem &p);
 size_t cooc_partial_words(int E);
 // bimg ([L][kBImageBytes], E = 128 only, may be null): the fp16 image of D'
@@ -205,6 +219,16 @@ cudaError_t launch_cooc_reduce(const uint32_t *partials, int P1, const int *n_ac
                                cudaStream_t s);
 
 // ---------------------------------------------------------------- device helpers
+
+// p advanced to the next multiple of A bytes of the shared window.  The offset
+// is added to p itself (no round trip through an integer), so the compiler
+// keeps every access through the result in the shared state space instead of
+// turning it into a generic access.
+template <uint32_t A>
+__device__ __forceinline__ unsigned char *smem_align(unsigned char *p) {
+    const uint32_t off = static_cast<uint32_t>(__cvta_generic_to_shared(p));
+    return p + ((A - (off & (A - 1u))) & (A - 1u));
+}
 
 __host__ __device__ __forceinline__ int64_t min64(int64_t a, int64_t b) { return a < b ? a : b; }
 

@@ -306,6 +306,25 @@ cudaError_t launch_loss(const float *logits, const uint32_t *bits, const int *D,
     return cudaGetLastError();
 }
 
+// Variance of the E (E - 1) off-diagonal distances of a local window from
+// Eq. origin_do (their sum of squares) and Eq. zero_sum (their sum is
+// 2 T k (E - k)): var = origin_do / (E (E - 1)) - mean^2 (App. C.1).  One
+// thread per problem, fp64.
+__global__ void offdiag_variance_kernel(const long long *__restrict__ origin_do, int64_t T, int E,
+                                        int k, int L, double *__restrict__ var) {
+    const int l = blockIdx.x * blockDim.x + threadIdx.x;
+    if (l >= L) return;
+    const double n = (double)E * (double)(E - 1);
+    const double mean = 2.0 * (double)T * (double)k * (double)(E - k) / n;
+    var[l] = (double)origin_do[l] / n - mean * mean;
+}
+
+cudaError_t launch_offdiag_variance(const long long *origin_do, const Problem &p, double *var,
+                                    cudaStream_t s) {
+    offdiag_variance_kernel<<<(p.L + 255) / 256, 256, 0, s>>>(origin_do, p.T, p.E, p.k, p.L, var);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_origin_do(const int *D, const Problem &p, long long *origin_do, cudaStream_t s) {
     origin_do_kernel<<<p.L, 256, 0, s>>>(D, p.E, origin_do);
     return cudaGetLastError();

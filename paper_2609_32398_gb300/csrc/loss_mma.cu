@@ -29,9 +29,8 @@
 //   warps 4-19   the epilogue: warp w reads TMEM lanes 32 (w % 4) .. +31 (its
 //                32 tokens) and the 32 experts of chunk (w - 4) / 4.  Each owns
 //                a 32 x 32 logits box per tile, loaded by TMA two tiles ahead;
-//                pass 1 forms s, S and SV and writes s (1 - s) and V back into
-//                the accumulator (the reciprocals of four 1 + e^-|z| in (1, 2]
-//                come from one rcp of their product); the four warps of a
+//                pass 1 forms s = 1 / (1 + e^-z), S and SV and writes s (1 - s)
+//                and V back into the accumulator; the four warps of a
 //                token quadrant exchange their (S, SV) through their boxes;
 //                pass 2 writes dz into the box in place and a TMA store sends
 //                it to dlogits; once the store has read the box it takes the
@@ -179,8 +178,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 loss_mma_kernel(const __grid_constant__ CUtensorMap zmap, const __grid_constant__ CUtensorMap dzmap,
                 const MmaArgs a) {
     extern __shared__ unsigned char smem_raw[];
-    unsigned char *smem = reinterpret_cast<unsigned char *>(
-        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    unsigned char *smem = smem_align<1024>(smem_raw);
     unsigned char *sB = smem + kOffB;
     unsigned char *sA = smem + kOffA;
     unsigned char *sZ = smem + kOffZ;
@@ -390,32 +388,19 @@ loss_mma_kernel(const __grid_constant__ CUtensorMap zmap, const __grid_constant_
                             z[4 * q + 3] = v.w;
                         }
                         tmem_wait_ld();
+                        // s = 1 / (1 + 2^(-z log2 e)): 0 when the power
+                        // overflows (z < -88), 1 when it underflows; the
+                        // Jacobian entry s (1 - s) as s - s^2 in one FMA (its
+                        // absolute error is an ulp of s, far below the
+                        // gradient's tolerance relative to its largest entry)
 #pragma unroll
-                        for (int g = 0; g < 4; ++g) {
-                            float ee[4], dd[4], inv[4];
-#pragma unroll
-                            for (int i = 0; i < 4; ++i) {
-                                ee[i] = ex2_approx(fabsf(z[4 * g + i]) * -kLog2e);
-                                dd[i] = 1.0f + ee[i];
-                            }
-                            const float p01 = dd[0] * dd[1], p012 = p01 * dd[2];
-                            float r = rcp_approx(p012 * dd[3]);
-                            inv[3] = r * p012;
-                            r *= dd[3];
-                            inv[2] = r * p01;
-                            r *= dd[2];
-                            inv[1] = r * dd[0];
-                            inv[0] = r * dd[1];
-#pragma unroll
-                            for (int i = 0; i < 4; ++i) {
-                                const int e = 4 * g + i;
-                                const float V = fmaf(__uint_as_float(hi[e]), 2048.0f, __uint_as_float(lo[e]));
-                                const float s = (z[e] >= 0.0f ? 1.0f : ee[i]) * inv[i];
-                                S += s;
-                                SV = fmaf(s, V, SV);
-                                hi[e] = __float_as_uint(ee[i] * inv[i] * inv[i]);
-                                lo[e] = __float_as_uint(V);
-                            }
+                        for (int e = 0; e < 16; ++e) {
+                            const float V = fmaf(__uint_as_float(hi[e]), 2048.0f, __uint_as_float(lo[e]));
+                            const float s = rcp_approx(1.0f + ex2_approx(z[e] * -kLog2e));
+                            S += s;
+                            SV = fmaf(s, V, SV);
+                            hi[e] = __float_as_uint(fmaf(-s, s, s));
+                            lo[e] = __float_as_uint(V);
                         }
                         tmem_st16(tl + 16 * h, hi);
                         tmem_st16(tl + kE + 16 * h, lo);

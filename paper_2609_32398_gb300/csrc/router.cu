@@ -26,8 +26,6 @@
 //            tokens), written out unpacked at the end; for longer ranges they
 //            go straight to the CTA's triangle in global memory as L2
 //            reductions.
-#include <cstdlib>
-#include <cstring>
 
 #include "sig_fast.cuh"
 
@@ -79,8 +77,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
 router_sig_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap wmap,
                   const __grid_constant__ CUtensorMap zmap, RouterArgs a) {
     extern __shared__ unsigned char smem_raw[];
-    unsigned char *smem = reinterpret_cast<unsigned char *>(
-        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    unsigned char *smem = smem_align<1024>(smem_raw);
     unsigned char *ring = smem;
     unsigned char *ztiles = smem + kROffZ;
     int *s_rowoff = reinterpret_cast<int *>(smem + kROffRowoff);
@@ -378,10 +375,8 @@ cudaError_t launch_router_signatures(const void *X, const void *Wr, int H, float
     a.H = H;
     const int ctas = router_ctas_per_problem(p);
     // 16-bit shared counters hold a CTA's counts while its range is below
-    // 65536 tokens; DOLOSS_ROUTER_COOC=global selects the L2 reductions
-    const char *mode = std::getenv("DOLOSS_ROUTER_COOC");
-    const bool force_global = mode && std::strcmp(mode, "global") == 0;
-    a.packed = !force_global && 32 * ((p.W + ctas - 1) / ctas) <= 65535;
+    // 65536 tokens; longer ranges add into the CTA's global triangle (L2)
+    a.packed = 32 * ((p.W + ctas - 1) / ctas) <= 65535;
     a.bits = bits;
     a.idx = idx;
     a.cooc = cooc;

@@ -12,8 +12,10 @@
 //      picks a group, the first element equal to its maximum is selected
 //      (lowest index among equal values), overwritten with -inf in shared
 //      memory, and the group maximum is recomputed.
-// The per-lane selections (a bit per expert) are turned into the signature
-// words of the 32 tokens by 32x32 bit transposes across the warp.
+// Each lane sets its token's bit in the words of its K chosen experts with
+// shared-memory atomic ORs into a per-warp scratch of E words, from which
+// lane c stores the words of experts c, c + 32, ... (the router kernel, whose
+// shared memory is full, builds the same words by 32x32 bit transposes).
 // The k selected indices of every token are also written (one byte each) for
 // the loss kernel, and the CTAs zero the accumulators of the next kernels.
 // The routing instantiations (kRoute) also write, per token, the chosen
@@ -47,7 +49,8 @@ struct SigCfg {
     // co-occurrence counters: row a holds columns (a & ~3) .. E-1
     static constexpr int kCoocWords = cooc_row_offset<E>(E);
     static constexpr size_t kSmem = (size_t)kSlots * kTileBytes + 1024 + 2 * kSlots * 8 +
-                                    kSlots * 4 + 32 + (size_t)kCoocWords * 4 + E * 4;
+                                    kSlots * 4 + 32 + (size_t)kCoocWords * 4 + E * 4 +
+                                    (size_t)kConsumers * E * 4;
 };
 
 
@@ -205,6 +208,28 @@ __device__ __forceinline__ void select_topk(unsigned char *tp, int lane, int (&s
     }
 }
 
+// Batcher's odd-even merge sort of K indices (K in {1, 2, 4, 8}) in registers.
+template <int K>
+__device__ __forceinline__ void sort_small(int (&so)[K]) {
+    auto cx = [&](int i, int j) {
+        const int lo = min(so[i], so[j]), hi = max(so[i], so[j]);
+        so[i] = lo;
+        so[j] = hi;
+    };
+    if constexpr (K == 2) {
+        cx(0, 1);
+    } else if constexpr (K == 4) {
+        cx(0, 1); cx(2, 3); cx(0, 2); cx(1, 3); cx(1, 2);
+    } else if constexpr (K == 8) {
+        cx(0, 1); cx(2, 3); cx(4, 5); cx(6, 7);
+        cx(0, 2); cx(1, 3); cx(4, 6); cx(5, 7);
+        cx(1, 2); cx(5, 6);
+        cx(0, 4); cx(1, 5); cx(2, 6); cx(3, 7);
+        cx(2, 4); cx(3, 5);
+        cx(1, 2); cx(3, 4); cx(5, 6);
+    }
+}
+
 // c_ab += 1 for every pair a < b of one token's chosen experts, in a
 // shared-memory triangle whose row a starts at s_rowoff[a] (the counts on the
 // diagonal come from the signature words).
@@ -213,14 +238,7 @@ __device__ __forceinline__ void cooc_add(uint32_t *s_cooc, const int *s_rowoff, 
     int so[K];
 #pragma unroll
     for (int q = 0; q < K; ++q) so[q] = sel[q];
-#pragma unroll
-    for (int i = 1; i < K; ++i)  // insertion sort of K indices (static network)
-#pragma unroll
-        for (int j = i; j > 0; --j) {
-            const int lo = min(so[j - 1], so[j]), hi = max(so[j - 1], so[j]);
-            so[j - 1] = lo;
-            so[j] = hi;
-        }
+    sort_small<K>(so);
 #pragma unroll
     for (int q1 = 0; q1 < K - 1; ++q1) {
         uint32_t *row = s_cooc + s_rowoff[so[q1]];
@@ -255,6 +273,30 @@ __device__ __forceinline__ void emit_words(const int (&sel)[K], bool valid, int 
     }
 }
 
+// The signature words of the warp's 32 tokens (lane = token) through the
+// warp's scratch s_w [E] (zero on entry and on return): every lane ORs its bit
+// into the words of its chosen experts, then lane c stores the words of
+// experts 32 r + c at words[(32 r + c) W].  With kCount, cnt[r] accumulates
+// the word's population count.
+template <int E, int K, bool kCount>
+__device__ __forceinline__ void emit_words_or(const int (&sel)[K], bool valid, int lane, uint32_t *s_w,
+                                              uint32_t *words, int64_t W, uint32_t (&cnt)[E / 32]) {
+    if (valid) {
+        const uint32_t bit = 1u << lane;
+#pragma unroll
+        for (int q = 0; q < K; ++q) atomicOr(s_w + sel[q], bit);
+    }
+    __syncwarp();
+#pragma unroll
+    for (int r = 0; r < E / 32; ++r) {
+        const uint32_t word = s_w[32 * r + lane];
+        s_w[32 * r + lane] = 0u;
+        words[(int64_t)(32 * r + lane) * W] = word;
+        if (kCount) cnt[r] += __popc(word);
+    }
+    __syncwarp();
+}
+
 template <int E, int K, bool kCounts, bool kCooc, bool kRoute>
 __global__ void __launch_bounds__(kFastThreads, 1)
 sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W,
@@ -263,8 +305,7 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W,
                 RouteOut route) {
     using C = SigCfg<E>;
     extern __shared__ unsigned char smem_raw[];
-    unsigned char *smem = reinterpret_cast<unsigned char *>(
-        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    unsigned char *smem = smem_align<1024>(smem_raw);
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + (size_t)C::kSlots * C::kTileBytes);
     uint64_t *empty = full + C::kSlots;
     // slot_round[s] = the round of slot s the producer has started to load.
@@ -274,8 +315,9 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W,
     volatile int *slot_round = reinterpret_cast<volatile int *>(empty + C::kSlots);
     volatile int *s_abort = slot_round + C::kSlots;
     uint32_t *s_cooc = reinterpret_cast<uint32_t *>(
-        (reinterpret_cast<uintptr_t>(s_abort + 1) + 15) & ~uintptr_t(15));
+        smem_align<16>(reinterpret_cast<unsigned char *>(const_cast<int *>(s_abort + 1))));
     int *s_rowoff = reinterpret_cast<int *>(s_cooc + C::kCoocWords);
+    uint32_t *s_wsc = reinterpret_cast<uint32_t *>(s_rowoff + E);  // [consumer warp][E]
 
     pdl_trigger();
     // this CTA: layer blockIdx.y, a contiguous range of its 32-token tiles
@@ -287,6 +329,7 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W,
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     // Shared-memory set-up first: it touches no global memory, so it overlaps
     // the end of the previous kernel on the stream.
+    for (int i = threadIdx.x; i < kConsumers * E; i += blockDim.x) s_wsc[i] = 0u;
     if (kCooc) {
         for (int i = threadIdx.x; i < C::kCoocWords; i += blockDim.x) s_cooc[i] = 0u;
         for (int a = threadIdx.x; a < E; a += blockDim.x) s_rowoff[a] = cooc_row_offset<E>(a) - (a & ~3);
@@ -381,7 +424,8 @@ sig_fast_kernel(const __grid_constant__ CUtensorMap tmap, int64_t T, int64_t W,
         if (idx && valid) store_idx<K>(idx + (layer * T + t) * K, sel);
         if (kRoute && valid) store_route<K>(route, (layer * T + t) * K, sel, val);
         if (kCooc && valid) cooc_add<K>(s_cooc, s_rowoff, sel);
-        emit_words<E, K, kCounts || kCooc>(sel, valid, lane, bits + layer * E * W + w, W, cnt);
+        emit_words_or<E, K, kCounts || kCooc>(sel, valid, lane, s_wsc + warp * E,
+                                             bits + layer * E * W + w, W, cnt);
     }
     if (kCounts) {
 #pragma unroll
@@ -428,8 +472,8 @@ cudaError_t run_fast(const CUtensorMap &map, const Problem &p, uint32_t *bits, i
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kern, map, p.T, p.W, bits, counts, idx, cooc, zero, status,
-                              route);
+    return cudaLaunchKernelEx(&cfg, kern, map, p.T, p.W, bits, counts, idx, cooc, zero,
+                              status, route);
 }
 
 template <int E, bool kCounts, bool kCooc, bool kRoute>

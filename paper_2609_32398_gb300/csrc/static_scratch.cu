@@ -11,6 +11,8 @@
 // The scratch is one array per device (one per CUDA context), so calls that
 // overlap in time — on two streams, or from two host threads — share it and
 // race; such callers must serialize their calls on one stream.
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
 #include <mutex>
@@ -24,26 +26,71 @@ constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) unsigned char g_scratch[DO_STATIC_SCRATCH_BYTES];
 
-std::mutex g_mu;
-void *g_scratch_ptr[kMaxDevices] = {};
+// The driver's current-context queries, reached through the runtime (the
+// library links no -lcuda).
+struct CtxFns {
+    PFN_cuCtxGetCurrent_v4000 current = nullptr;
+    PFN_cuCtxGetId_v12000 id = nullptr;
+};
 
-// Address of the scratch on the current device.  The first call on a device
-// looks it up (the device must be current, as it is here) and zero-fills it,
-// then waits for the device so that the fill is complete before any stream
-// uses the array.
+const CtxFns &ctx_fns() {
+    static CtxFns f;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) ==
+                cudaSuccess && q == cudaDriverEntryPointSuccess)
+            f.current = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(p);
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess && q == cudaDriverEntryPointSuccess)
+            f.id = reinterpret_cast<PFN_cuCtxGetId_v12000>(p);
+    });
+    return f;
+}
+
+// Identifier of the current context (unique for the life of the process,
+// never reused), 0 if none is current or the query is unavailable.
+unsigned long long current_ctx_id() {
+    const CtxFns &f = ctx_fns();
+    CUcontext ctx = nullptr;
+    unsigned long long id = 0;
+    if (f.current && f.id && f.current(&ctx) == CUDA_SUCCESS && ctx && f.id(ctx, &id) == CUDA_SUCCESS)
+        return id;
+    return 0;
+}
+
+std::mutex g_mu;
+struct Cached {
+    unsigned long long ctx;
+    void *ptr;
+};
+Cached g_cache[kMaxDevices] = {};
+
+// Device address of the scratch array in the current context.  In host code
+// the name g_scratch stands for a host-side shadow, not a device address, so
+// the address is looked up with cudaGetSymbolAddress, with the device current.
+// The lookup is cached per device and keyed by the context's identifier: a
+// context created after cudaDeviceReset (or after the primary context was
+// released) holds a new copy of the module, and its first call looks up the
+// address again.  The first call in a context therefore does this set-up; it
+// should come before any stream capture begins.
 do_status scratch_on_current_device(void **out) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return DO_ERR_CUDA;
     if (dev < 0 || dev >= kMaxDevices) return DO_ERR_UNSUPPORTED;
     std::lock_guard<std::mutex> lock(g_mu);
-    if (!g_scratch_ptr[dev]) {
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_scratch) != cudaSuccess || !p) return DO_ERR_CUDA;
-        if (cudaMemset(p, 0, DO_STATIC_SCRATCH_BYTES) != cudaSuccess) return DO_ERR_CUDA;
-        if (cudaDeviceSynchronize() != cudaSuccess) return DO_ERR_CUDA;
-        g_scratch_ptr[dev] = p;
+    const unsigned long long ctx = current_ctx_id();
+    if (ctx != 0 && g_cache[dev].ctx == ctx && g_cache[dev].ptr) {
+        *out = g_cache[dev].ptr;
+        return DO_OK;
     }
-    *out = g_scratch_ptr[dev];
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_scratch) != cudaSuccess || !p) return DO_ERR_CUDA;
+    // the lookup makes the device's primary context current if none was
+    g_cache[dev].ctx = ctx != 0 ? ctx : current_ctx_id();
+    g_cache[dev].ptr = p;
+    *out = p;
     return DO_OK;
 }
 
@@ -77,13 +124,14 @@ extern "C" do_status do_forward_backward_static(const float *logits, int64_t T, 
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     // What must be zero when a call starts: the status word and the done
     // counters (the first 256-byte-aligned span) and the counts accumulator
-    // (the last span).  The kernels leave them zero after a complete call;
+    // [n_acc, bimg).  The kernels leave them zero after a complete call;
     // clearing them here also recovers from a call that gave up on a wait.
+    // Everything else in the array is written before it is read (the image
+    // of D' at bimg by the reduction kernel, every entry of it).
     const dol::WsLayout w = dol::ws_layout(p);
     char *base = static_cast<char *>(ws);
     if (cudaMemsetAsync(base, 0, w.partials, s) != cudaSuccess) return DO_ERR_CUDA;
-    if (w.route_base > w.n_acc &&
-        cudaMemsetAsync(base + w.n_acc, 0, w.route_base - w.n_acc, s) != cudaSuccess)
+    if (w.bimg > w.n_acc && cudaMemsetAsync(base + w.n_acc, 0, w.bimg - w.n_acc, s) != cudaSuccess)
         return DO_ERR_CUDA;
     st = do_forward_backward(logits, T, E, k, L, gate, grad_scale, bits, counts, D, loss, origin_do,
                              dlogits, ws, DO_STATIC_SCRATCH_BYTES, stream);

@@ -48,6 +48,7 @@ EXPORTS = {
     "do_route_backward": (["p", "p", "p", "i64", "i32", "i32", "i32", "i32", "i32", "p", "p", "p"],
                           "i32"),
     "do_accumulate_distances": (["p", "i32", "i32", "p", "p"], "i32"),
+    "do_offdiag_variance": (["p", "i64", "i32", "i32", "i32", "p", "p"], "i32"),
     "do_routed_forward": (["p", "i64", "i32", "i32", "i32", "i32", "p", "p", "p", "p", "p", "p", "p",
                            "p", "p", "p", "sz", "p"], "i32"),
     "do_routed_backward": (["p", "i64", "i32", "i32", "i32", "i32", "f32", "f32", "p", "p", "p", "p",
@@ -668,13 +669,14 @@ def route(logits: torch.Tensor, k: int, gate=GATE_SIGMOID_NORM):
     return _RouteFunction.apply(logits, k, gate)
 
 
-def offdiag_variance(origin_do, T: int, E: int, k: int):
-    """Variance of the off-diagonal entries of a local Hamming matrix, from
-    Eq. origin_do (the exact sum of their squares) and Eq. zero_sum (their sum
-    is 2 T k (E - k)): Var = origin_do / (E (E - 1)) - mean^2.  origin_do may
-    be an int, or an int64 tensor [L] (returned as float64 [L])."""
-    n = E * (E - 1)
-    mean = 2.0 * T * k * (E - k) / n
-    if isinstance(origin_do, torch.Tensor):
-        return origin_do.double() / n - mean * mean
-    return int(origin_do) / n - mean * mean
+def offdiag_variance(origin_do: torch.Tensor, T: int, E: int, k: int) -> torch.Tensor:
+    """do_offdiag_variance: the variance of the off-diagonal entries of each
+    problem's local Hamming matrix (App. C.1) from origin_do [L] int64 (CUDA),
+    computed on the device; returns float64 [L]."""
+    if origin_do.dtype != torch.int64 or not origin_do.is_cuda or not origin_do.is_contiguous():
+        raise ValueError("origin_do must be a contiguous CUDA int64 tensor")
+    L = origin_do.numel()
+    var = torch.empty(L, dtype=torch.float64, device=origin_do.device)
+    _check("do_offdiag_variance", lib().do_offdiag_variance(
+        origin_do.data_ptr(), T, E, k, L, var.data_ptr(), _stream(origin_do)))
+    return var
