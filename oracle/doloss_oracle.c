@@ -176,7 +176,9 @@ void oracle_dloss_dp(const int32_t *D, const uint8_t *f, int64_t t0, int64_t t1,
 
 /* Chain rule through the router gate, with the Jacobian written out entry by
  * entry: dz_lt = grad_scale * sum_i (d p_it / d z_lt) g_it.
- *  sigmoid-norm: d p_i / d z_l = (delta_il - p_i) / S * s_l (1 - s_l), S = sum s
+ *  sigmoid-norm: d p_i / d z_l = (delta_il - p_i) / S * s_l (1 - s_l), S = sum s,
+ *                with 1 - s_l evaluated as sigmoid(-z_l) (no cancellation for
+ *                large z_l)
  *  softmax:      d p_i / d z_l = p_i (delta_il - p_l)                          */
 void oracle_gate_backward(const float *z, const double *g, int64_t t0, int64_t t1,
                           int32_t E, int32_t gate, double grad_scale, double *dz)
@@ -197,7 +199,7 @@ void oracle_gate_backward(const float *z, const double *g, int64_t t0, int64_t t
                 if (gate == GATE_SOFTMAX)
                     J = p[i] * (delta - p[l]);
                 else
-                    J = (delta - p[i]) / S * s[l] * (1.0 - s[l]);
+                    J = (delta - p[i]) / S * s[l] * (1.0 / (1.0 + exp((double)zt[l])));
                 acc += J * gt[i];
             }
             dz[t * E + l] = grad_scale * acc;

@@ -236,6 +236,35 @@ def test_gradient_matches_torch_autograd(gk):
     assert oracle.loss(D, C, T, k, d_scale=0.75) == pytest.approx(L.item(), rel=1e-12)
 
 
+@pytest.mark.parametrize("zbig", [40.0, 60.0, -60.0])
+def test_sigmoid_gate_backward_at_saturated_logits(zbig):
+    """Sigmoid-norm gate backward where s is within 1e-17 of 1 (or of 0): the
+    Jacobian factor s (1 - s) must come out as sigmoid(z) sigmoid(-z), not as
+    the cancelled 1 - s.  Pinned to a 50-digit numerical derivative of
+    p_i(z) = s_i / sum_j s_j (mpmath), independent of the oracle's formula."""
+    mpmath = pytest.importorskip("mpmath")
+    mp = mpmath.mp
+    mp.dps = 50
+    z = np.array([[zbig, 0.5, -1.0, 2.0]], np.float32)
+    g = np.array([[1.5, -0.25, 0.75, 0.0]], np.float64)
+    dz = oracle.gate_backward(z, g, oracle.GATE_SIGMOID_NORM, grad_scale=1.0)[0]
+
+    def p_dot_g(zz):
+        s = [1 / (1 + mpmath.exp(-v)) for v in zz]
+        S = sum(s)
+        return sum(mpmath.mpf(float(g[0, i])) * s[i] / S for i in range(4))
+
+    zm = [mpmath.mpf(float(v)) for v in z[0]]
+    for l in range(4):
+        def along(h, l=l):
+            zz = list(zm)
+            zz[l] = zz[l] + h
+            return p_dot_g(zz)
+        want = float(mpmath.diff(along, 0))
+        assert dz[l] == pytest.approx(want, rel=1e-12, abs=1e-300), (l, dz[l], want)
+    assert dz[0] != 0.0
+
+
 def test_straight_through_gradient_is_four_times_surrogate():
     """Sec. 3.1.2: with F_i -> P_i + sg[F_i - P_i], the origin loss keeps the value
     sum_{i!=j} ||F_i - F_j||^2 (Eq. origin_do) and its gradient in p_it is
@@ -377,14 +406,3 @@ def test_dense_p_reading_against_the_renormalized_one():
     C1 = oracle.direction_mode(z, f, mode=1)
     assert C1.sum() == pytest.approx(T * (E - k), rel=1e-12)
 
-
-def test_offdiag_variance_from_origin_do():
-    """Eq. origin_do with Eq. zero_sum gives the variance of the off-diagonal
-    distances without reading D (numpy's variance of the entries pins it)."""
-    from paper_2609_32398_gb300.doloss import offdiag_variance
-
-    for T, E, k in ((97, 8, 2), (500, 33, 5)):
-        f = oracle.select(rand_z(T, E, T + E), k)
-        D = oracle.hamming(f)
-        off = D[~np.eye(E, dtype=bool)].astype(np.float64)
-        assert offdiag_variance(oracle.origin_do(D), T, E, k) == pytest.approx(off.var(), rel=1e-12)

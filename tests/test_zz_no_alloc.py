@@ -29,10 +29,16 @@ def test_static_scratch_matches_workspace_path(dl, T, E, k, L, gate):
     ref = dl.forward_backward(z, k, gate, grad_scale=1.5)
     assert dl.device_status(ref.workspace) == 0
     flags = torch.full((1,), -1, dtype=torch.int32, device="cuda")
-    for _ in range(2):  # two consecutive calls on the same scratch
-        out = dl.Buffers(L, T, E, k, "cuda")
+    outs = [dl.Buffers(L, T, E, k, "cuda") for _ in range(2)]
+    for i in range(2):  # two consecutive calls on the same scratch
+        out = outs[i]
+        torch.cuda.synchronize()
+        free0, allocated0 = torch.cuda.mem_get_info()[0], torch.cuda.memory_allocated()
         dl.forward_backward_static(z, k, out, gate, grad_scale=1.5, status_flags=flags)
         torch.cuda.synchronize()
+        if i > 0:  # the first call in the process may load the module's code
+            assert torch.cuda.mem_get_info()[0] == free0, "device memory was allocated"
+        assert torch.cuda.memory_allocated() == allocated0
         assert int(flags[0]) == 0
         for name in ("bits", "counts", "D", "origin_do"):
             assert torch.equal(getattr(out, name), getattr(ref, name)), name
