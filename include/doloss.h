@@ -26,9 +26,8 @@
  *  - Every array argument is a DEVICE pointer owned by the caller, except in
  *    do_forward_backward_host(_async), whose h_* arguments are host pointers,
  *    and do_rem_allocate, a host function.  The library allocates nothing and
- *    keeps no state between calls, with two stated exceptions:
- *    do_forward_backward_static (a fixed scratch array per device) and
- *    do_router_backward (a cuBLAS handle per device).  do_routed_backward
+ *    keeps no state between calls, with one stated exception:
+ *    do_forward_backward_static (a fixed scratch array per device).  do_routed_backward
  *    reads what do_routed_forward left in the caller's workspace.
  *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default
  *    stream).  Calls are asynchronous on it, except do_device_status and
@@ -299,15 +298,15 @@ do_status do_router_forward_backward(const void *X, const void *Wr, int64_t T, i
  *   dW [L][E][H] fp32,  dW[l][e][h] = sum_t dz[l][t][e] X[l][t][h]
  *   dX [L][T][H] bf16,  dX[l][t][h] = sum_e dz[l][t][e] W[l][e][h]  (may be NULL)
  * X, W bf16 as in do_router_forward_backward; all arrays 16-byte aligned.
- * dz is rounded to bf16 (nearest even) by the library and both products run
- * in cuBLAS (bf16 inputs, fp32 accumulation): plain matrix products with the
- * reduction index outermost in memory.  cuBLAS is opened at run time; where
- * it cannot be, the call returns DO_ERR_UNSUPPORTED.  Unlike the other entry
- * points this one keeps state: the first call on a device creates a cuBLAS
- * handle for it, and calls are serialised on a lock.  workspace:
+ * E = 128 and H a multiple of 64 (DO_ERR_UNSUPPORTED otherwise).  dz is
+ * rounded to bf16 (nearest even) and both products run on the tensor cores
+ * (bf16 operands, fp32 accumulation; X, W and dz read as stored); dW is the
+ * sum of per-chunk partial products over the tokens, added in a fixed order,
+ * so results are identical run to run.  workspace:
  * do_router_backward_workspace_size bytes of device memory, 256-byte
- * aligned (the bf16 copy of dz and cuBLAS's workspace).  T <= INT32_MAX and
- * E H <= INT32_MAX.  Asynchronous on `stream`. */
+ * aligned and zero-filled before its first use (its status word, read by
+ * do_device_status; then the bf16 copy of dz and the partial sums).
+ * Asynchronous on `stream`. */
 do_status do_router_backward(const void *X, const void *Wr, const float *dlogits, int64_t T,
                              int32_t H, int32_t E, int32_t L, float *dW, void *dX,
                              void *workspace, size_t workspace_bytes, void *stream);

@@ -1,30 +1,43 @@
 // Step 2: the detached Hamming matrix of the load signatures.
 //   G_ij = ||F_i - F_j||_1 = sum over words of popc(F_i[w] XOR F_j[w])
-//   (Sec. 3.1.3, Eq. gij_cij)
-// A CTA owns a 16 x 16 tile of expert pairs on or above the diagonal and a
-// chunk of signature words; it stages both row blocks of the chunk in shared
-// memory and adds its exact integer partial sums into D (zeroed beforehand),
-// so the result does not depend on the order in which chunks finish.  On the
-// diagonal tiles the threads of pairs (i, i) count the set bits of F_i
-// instead, which gives the per-expert counts n_i = ||F_i||_1 (App. C.3).
+//   (Sec. 3.1.3, Eq. gij_cij; App. C.3: n_i = ||F_i||_1)
+// A CTA owns an 8 x 8 block of expert pairs on or above the diagonal and all
+// the signature words, so every entry of D has one writer: no atomics and no
+// clearing beforehand.  Its 256 threads split the words 64 ways (a
+// contiguous slice each) and hold 4 x 4 pairs in registers (a quarter of the
+// block), so every 16-byte load of a row feeds four pairs; the 64 slices'
+// partial sums are added in shared memory in a fixed order.
 #include "dol_internal.cuh"
 #include "tma.cuh"
 
 namespace dol {
 namespace {
 
-constexpr int kTile = 16;            // experts per tile side
-constexpr int kPass = 256;           // words staged per pass
-constexpr int kStride = kPass + 4;   // padded row stride (keeps 16-byte loads conflict-free)
-constexpr int kHamThreads = kTile * kTile;
+constexpr int kHB = 8;        // experts per block side
+constexpr int kHSlices = 64;  // word slices per block
+constexpr int kHThreads = kHSlices * 4;
 
-__global__ void __launch_bounds__(kHamThreads)
-hamming_kernel(const uint32_t *__restrict__ bits, int E, int64_t W, int nside, int64_t chunk_words,
-               int *__restrict__ D, int *__restrict__ counts, int vec) {
-    __shared__ __align__(16) uint32_t s_a[kTile * kStride];
-    __shared__ __align__(16) uint32_t s_b[kTile * kStride];
+__device__ __forceinline__ uint4 load_w4(const uint32_t *row, int64_t w, int64_t w_end, bool vec) {
+    if (!row) return make_uint4(0u, 0u, 0u, 0u);
+    if (vec && w + 4 <= w_end) return __ldg(reinterpret_cast<const uint4 *>(row + w));
+    uint32_t q[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) q[i] = (w + i < w_end) ? __ldg(row + w + i) : 0u;
+    return make_uint4(q[0], q[1], q[2], q[3]);
+}
 
-    // Upper-triangle tile index -> (bi, bj), bi <= bj.
+__device__ __forceinline__ int popc_xor4(uint4 a, uint4 b) {
+    return __popc(a.x ^ b.x) + __popc(a.y ^ b.y) + __popc(a.z ^ b.z) + __popc(a.w ^ b.w);
+}
+
+// accumulate: D (and counts, when given) += the result; else D = the result
+// (and counts = n).
+__global__ void __launch_bounds__(kHThreads)
+hamming_kernel(const uint32_t *__restrict__ bits, int E, int64_t W, int nside, int *__restrict__ D,
+               int *__restrict__ counts, int accumulate, int vec) {
+    __shared__ int s_part[kHSlices][kHB * kHB];
+    __shared__ int s_cnt[kHSlices][kHB];
+    // upper-triangle block index -> (bi, bj), bi <= bj
     int t = blockIdx.x, bi = 0;
     while (t >= nside - bi) {
         t -= nside - bi;
@@ -33,95 +46,88 @@ hamming_kernel(const uint32_t *__restrict__ bits, int E, int64_t W, int nside, i
     const int bj = bi + t;
     const int layer = blockIdx.z;
     const uint32_t *bl = bits + (int64_t)layer * E * W;
-    const int64_t w_begin = (int64_t)blockIdx.y * chunk_words;
-    const int64_t w_end = min64(W, w_begin + chunk_words);
-    const int ti = threadIdx.x / kTile, tj = threadIdx.x % kTile;
-    const int I = bi * kTile + ti, J = bj * kTile + tj;
-    const bool count_row = (bi == bj) && (ti == tj);
-    // staging: thread -> (row, 16-byte column) of both row blocks
-    const int srow = threadIdx.x >> 4, scol = (threadIdx.x & 15) * 4;
-    const int ra = bi * kTile + srow, rb = bj * kTile + srow;
-
+    const int sl = threadIdx.x >> 2, sb = threadIdx.x & 3;
+    const int ri0 = 4 * (sb >> 1), cj0 = 4 * (sb & 1);  // this thread's 4 rows and 4 columns
+    // words of this slice: a multiple of 4 per slice
+    const int64_t per = ((W + kHSlices - 1) / kHSlices + 3) / 4 * 4;
+    const int64_t w0 = (int64_t)sl * per, w1 = min64(W, w0 + per);
+    const uint32_t *ra[4], *rb[4];
+#pragma unroll
+    for (int x = 0; x < 4; ++x) {
+        const int i = kHB * bi + ri0 + x, j = kHB * bj + cj0 + x;
+        ra[x] = i < E ? bl + (int64_t)i * W : nullptr;
+        rb[x] = j < E ? bl + (int64_t)j * W : nullptr;
+    }
+    const bool diag_counts = counts && bi == bj && sb == 0;  // rows 0..3 ...
+    const bool diag_counts2 = counts && bi == bj && sb == 3; // ... and rows 4..7 of a diagonal block
     pdl_wait();
     pdl_trigger();
-    int acc = 0;
-    for (int64_t w0 = w_begin; w0 < w_end; w0 += kPass) {
-        const int nw = (int)min64(kPass, w_end - w0);
-        __syncthreads();
+    int acc[4][4];
 #pragma unroll
-        for (int c0 = 0; c0 < kPass; c0 += 64) {
-            const int c = c0 + scol;
-            uint4 va = make_uint4(0u, 0u, 0u, 0u), vb = va;
-            if (c < nw) {
-                const uint32_t *pa = bl + (int64_t)ra * W + w0 + c;
-                const uint32_t *pb = bl + (int64_t)rb * W + w0 + c;
-                if (vec && c + 4 <= nw) {
-                    if (ra < E) va = __ldg(reinterpret_cast<const uint4 *>(pa));
-                    if (rb < E) vb = __ldg(reinterpret_cast<const uint4 *>(pb));
-                } else {
-                    uint32_t a4[4] = {0u, 0u, 0u, 0u}, b4[4] = {0u, 0u, 0u, 0u};
-                    for (int q = 0; q < 4 && c + q < nw; ++q) {
-                        if (ra < E) a4[q] = __ldg(pa + q);
-                        if (rb < E) b4[q] = __ldg(pb + q);
-                    }
-                    va = make_uint4(a4[0], a4[1], a4[2], a4[3]);
-                    vb = make_uint4(b4[0], b4[1], b4[2], b4[3]);
-                }
-            }
-            *reinterpret_cast<uint4 *>(s_a + srow * kStride + c) = va;
-            *reinterpret_cast<uint4 *>(s_b + srow * kStride + c) = vb;
+    for (int x = 0; x < 4; ++x)
+#pragma unroll
+        for (int y = 0; y < 4; ++y) acc[x][y] = 0;
+    int cnt[4] = {0, 0, 0, 0};
+    for (int64_t w = w0; w < w1; w += 4) {
+        uint4 a[4], b[4];
+#pragma unroll
+        for (int x = 0; x < 4; ++x) {
+            a[x] = load_w4(ra[x], w, w1, vec);
+            b[x] = load_w4(rb[x], w, w1, vec);
         }
-        __syncthreads();
-        const uint4 *pa = reinterpret_cast<const uint4 *>(s_a + ti * kStride);
-        const uint4 *pb = reinterpret_cast<const uint4 *>(s_b + tj * kStride);
-        const int n4 = (nw + 3) >> 2;
-        if (count_row) {
-            for (int c = 0; c < n4; ++c) {
-                const uint4 a = pa[c];
-                acc += __popc(a.x) + __popc(a.y) + __popc(a.z) + __popc(a.w);
-            }
-        } else {
-            for (int c = 0; c < n4; ++c) {
-                const uint4 a = pa[c], b = pb[c];
-                acc += __popc(a.x ^ b.x) + __popc(a.y ^ b.y) + __popc(a.z ^ b.z) + __popc(a.w ^ b.w);
-            }
+#pragma unroll
+        for (int x = 0; x < 4; ++x)
+#pragma unroll
+            for (int y = 0; y < 4; ++y) acc[x][y] += popc_xor4(a[x], b[y]);
+        if (diag_counts || diag_counts2) {
+#pragma unroll
+            for (int x = 0; x < 4; ++x)
+                cnt[x] += __popc(a[x].x) + __popc(a[x].y) + __popc(a[x].z) + __popc(a[x].w);
         }
     }
-    if (count_row) {
-        if (counts && I < E && acc) atomicAdd(counts + (int64_t)layer * E + I, acc);
-        return;
-    }
-    const bool pair = (I < E) && (J < E) && (bi != bj || ti < tj);
-    if (pair && acc) {
-        int *Dl = D + (int64_t)layer * E * E;
-        atomicAdd(Dl + (int64_t)I * E + J, acc);
-        atomicAdd(Dl + (int64_t)J * E + I, acc);
+#pragma unroll
+    for (int x = 0; x < 4; ++x)
+#pragma unroll
+        for (int y = 0; y < 4; ++y) s_part[sl][(ri0 + x) * kHB + cj0 + y] = acc[x][y];
+    if (diag_counts || diag_counts2)
+#pragma unroll
+        for (int x = 0; x < 4; ++x) s_cnt[sl][ri0 + x] = cnt[x];
+    __syncthreads();
+    // the 64 pairs of the block, each the fixed-order sum over the slices
+    if (threadIdx.x < kHB * kHB) {
+        const int ii = threadIdx.x / kHB, jj = threadIdx.x % kHB;
+        const int i = kHB * bi + ii, j = kHB * bj + jj;
+        if (i < E && j < E && (bi != bj || ii < jj)) {
+            int d = 0;
+            for (int v = 0; v < kHSlices; ++v) d += s_part[v][threadIdx.x];
+            int *Dl = D + (int64_t)layer * E * E;
+            if (accumulate) {
+                Dl[(int64_t)i * E + j] += d;
+                Dl[(int64_t)j * E + i] += d;
+            } else {
+                Dl[(int64_t)i * E + j] = d;
+                Dl[(int64_t)j * E + i] = d;
+            }
+        }
+        if (bi == bj && ii == jj && i < E) {
+            if (!accumulate) D[(int64_t)layer * E * E + (int64_t)i * E + i] = 0;
+            if (counts) {
+                int n = 0;
+                for (int v = 0; v < kHSlices; ++v) n += s_cnt[v][ii];
+                int *dst = counts + (int64_t)layer * E + i;
+                *dst = accumulate ? *dst + n : n;
+            }
+        }
     }
 }
 
-}  // namespace
-
-// D (and counts, when given) must be zero when the kernel starts; the caller
-// either memsets them or has the preceding kernel clear them.
-cudaError_t launch_hamming_accumulate(const uint32_t *bits, const Problem &p, int *D, int *counts,
-                                      cudaStream_t s) {
-    const int nside = (p.E + kTile - 1) / kTile;
-    const int ntiles = nside * (nside + 1) / 2;
-    int dev = 0, sms = 148;
-    if (cudaGetDevice(&dev) == cudaSuccess)
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    // Split the words so that one launch fills the GPU about twice.
-    int64_t target = (2LL * sms + (int64_t)ntiles * p.L - 1) / ((int64_t)ntiles * p.L);
-    if (target < 1) target = 1;
-    int64_t max_chunks = (p.W + 63) / 64;
-    if (max_chunks < 1) max_chunks = 1;
-    const int64_t nchunks = target < max_chunks ? target : max_chunks;
-    int64_t chunk = (p.W + nchunks - 1) / nchunks;
-    chunk = (chunk + 3) / 4 * 4;
-    const int64_t gy = (p.W + chunk - 1) / chunk;
+cudaError_t run_hamming(const uint32_t *bits, const Problem &p, int *D, int *counts, int accumulate,
+                        cudaStream_t s) {
+    const int nside = (p.E + kHB - 1) / kHB;
+    const int nblocks = nside * (nside + 1) / 2;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)ntiles, (unsigned)gy, (unsigned)p.L);
-    cfg.blockDim = dim3(kHamThreads);
+    cfg.gridDim = dim3((unsigned)nblocks, 1u, (unsigned)p.L);
+    cfg.blockDim = dim3(kHThreads);
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -129,13 +135,19 @@ cudaError_t launch_hamming_accumulate(const uint32_t *bits, const Problem &p, in
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     const int vec = (p.W % 4 == 0) && (reinterpret_cast<uintptr_t>(bits) % 16 == 0);
-    return cudaLaunchKernelEx(&cfg, hamming_kernel, bits, p.E, p.W, nside, chunk, D, counts, vec);
+    return cudaLaunchKernelEx(&cfg, hamming_kernel, bits, p.E, p.W, nside, D, counts, accumulate, vec);
+}
+
+}  // namespace
+
+// D (and counts, when given) += the Hamming matrix of bits (and the counts).
+cudaError_t launch_hamming_accumulate(const uint32_t *bits, const Problem &p, int *D, int *counts,
+                                      cudaStream_t s) {
+    return run_hamming(bits, p, D, counts, 1, s);
 }
 
 cudaError_t launch_hamming(const uint32_t *bits, const Problem &p, int *D, cudaStream_t s) {
-    cudaError_t e = cudaMemsetAsync(D, 0, sizeof(int) * (size_t)p.L * p.E * p.E, s);
-    if (e != cudaSuccess) return e;
-    return launch_hamming_accumulate(bits, p, D, nullptr, s);
+    return run_hamming(bits, p, D, nullptr, 0, s);
 }
 
 // D_sum += D over n int32 entries (the Hamming matrices of the micro-batches

@@ -411,7 +411,7 @@ def router_backward(X: torch.Tensor, Wr: torch.Tensor, dlogits: torch.Tensor, wi
     dW = torch.empty(L, E, H, dtype=torch.float32, device=X.device)
     dX = torch.empty(L, T, H, dtype=torch.bfloat16, device=X.device) if with_dx else None
     if workspace is None:
-        workspace = torch.empty(int(lib().do_router_backward_workspace_size(T, E, H, L)),
+        workspace = torch.zeros(int(lib().do_router_backward_workspace_size(T, E, H, L)),
                                 dtype=torch.uint8, device=X.device)
     _check("do_router_backward", lib().do_router_backward(
         X.data_ptr(), Wr.data_ptr(), dz.data_ptr(), T, H, E, L, dW.data_ptr(), _ptr(dX),
