@@ -300,6 +300,45 @@ def run_reference(args, rank, world):
     print(json.dumps(line), flush=True)
 
 
+# The other workloads of the path (the 4.8BA0.5B-shaped layer, the collapse
+# regime and the 30BA3B-depth long window, 48 layers in one call), each timed
+# through do_forward_backward with enough rotating buffer sets that the sets
+# exceed L2 twice over (the larger ones exceed it on their own).
+OTHER_WORKLOADS = {"c2": 500, "collapse": 200, "long": 3}  # calls timed
+L2_BYTES = 129 * 2**20
+
+
+def time_workload(dl, torch, workloads, name, reps, dev):
+    """Microseconds per do_forward_backward call on the workload `name`."""
+    w = workloads.get(name)
+    per_set = 8 * w.T * w.E * w.L
+    n_sets = max(1, -(-2 * L2_BYTES // per_set))
+    base = workloads.logits(w, dev)
+    sets = [(base if s == 0 else base + 0.0, dl.Buffers(w.L, w.T, w.E, w.k, dev))
+            for s in range(n_sets)]
+
+    def call(i):
+        z, out = sets[i % n_sets]
+        dl.forward_backward(z, w.k, w.gate, 1.0, out=out)
+
+    for i in range(max(3, n_sets)):
+        call(i)
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record()
+    for i in range(reps):
+        call(i)
+    ev1.record()
+    torch.cuda.synchronize()
+    us = ev0.elapsed_time(ev1) * 1e3 / reps
+    st = dl.device_status(sets[0][1].workspace)
+    if st != 0:
+        raise RuntimeError(f"device status after the {name} runs: {dl.status_string(st)}")
+    del sets, base
+    torch.cuda.empty_cache()
+    return w, us, n_sets
+
+
 def config_dict(w):
     return {"workload": f"3B-active-shaped router layer: E={w.E} k={w.k} T={w.T} L={w.L}",
             "E": w.E, "k": w.k, "T": w.T, "L": w.L, "gate": "sigmoid_norm",
@@ -576,7 +615,7 @@ def run_ours(args, rank, world, local):
     st = dl.device_status(rout.workspace)
     if st != 0:
         raise RuntimeError(f"device status after the router runs: {dl.status_string(st)}")
-    # the router's backward (dz -> bf16 in our kernel, dW and dX in cuBLAS)
+    # the router's backward (dz -> bf16, dW and dX on the tensor cores in our kernels)
     rbw = torch.empty(int(dl.lib().do_router_backward_workspace_size(T, E, ROUTER_HIDDEN, L)),
                       dtype=torch.uint8, device=dev)
     for _ in range(3):
@@ -600,6 +639,18 @@ def run_ours(args, rank, world, local):
 
     peaks = measured_peaks()
     peak = peaks["hbm_gbs"] if peaks else 6800.0
+    others = {}
+    for name, reps_w in OTHER_WORKLOADS.items():
+        ow, us, n_sets = time_workload(dl, torch, workloads, name, reps_w, dev)
+        ab = algorithmic_bytes(ow.T, ow.E, ow.L)
+        others[name] = {
+            "workload": ow.describe(), "us_per_call": us,
+            "tokens_per_s": ow.T * ow.L / (us * 1e-6),
+            "roofline": {"bound": "hbm", "achieved": ab / (us * 1e-6) / 1e9, "peak": peak,
+                         "unit": "GB/s", "frac": ab / (us * 1e-6) / 1e9 / peak,
+                         "peak_source": "of measured" if peaks else "of fallback",
+                         "algorithmic_bytes": ab},
+            "buffer_sets": n_sets, "calls": reps_w}
     peak_src = "of measured" if peaks else "of fallback"
     # The unit of the roofline is one do_forward_backward launch sequence (three
     # dependent kernels chained by programmatic dependent launch), timed by the
@@ -658,6 +709,9 @@ def run_ours(args, rank, world, local):
                 raise RuntimeError(f"device status flags {flags} in the pipelined host calls")
         e2e = {"value": rate_pipe, "unit": UNIT, "h2d_bytes_per_step": 4 * T * E * L,
                "d2h_bytes_per_step": 4 * L + 4, "ms_per_step": dt_pipe * 1e3,
+               "read_back": "the losses and the device status word; dlogits are computed every "
+                            "step and kept in device memory (with_dlogits_to_host copies them "
+                            "out as well)",
                "api": "do_forward_backward_host_async, two device buffers and two streams",
                "synchronous_calls": {"value": rate, "d2h_bytes_per_step": 4 * L + 4,
                                      "ms_per_step": dt * 1e3,
@@ -762,12 +816,13 @@ def run_ours(args, rank, world, local):
                              "traffic": profiled_traffic("do_router_forward_backward")},
                 "context_unfused_us": {"cublas_bf16_matmul": cublas_ms * 1e3,
                                        "do_forward_backward": plain_ms * 1e3},
-                "backward": {"entry": "do_router_backward (dz rounded to bf16 by our kernel; dW "
-                                      "fp32 and dX bf16 by cuBLAS)",
+                "backward": {"entry": "do_router_backward (dz rounded to bf16; dW fp32 and dX "
+                                      "bf16 by tcgen05 kernels)",
                              "us_per_call": router_bwd_ms * 1e3,
                              "bytes": 2 * T * L * ROUTER_HIDDEN * 2 + 4 * T * E * L + 4 * T * E * L
                              + 2 * E * ROUTER_HIDDEN * L + 4 * E * ROUTER_HIDDEN * L},
                 "reps": router_reps},
+            "other_workloads": others,
             "clocks": clocks, "e2e": e2e, "gpu_launches": KERNELS_PER_STEP * args.steps,
             "cpu_baseline": cpu,
         }
