@@ -740,6 +740,9 @@ def run_ours(args, rank, world, local):
                          "frac": achieved / peak, "peak_source": peak_src,
                          "algorithmic_bytes": algorithmic_bytes(T, E, L),
                          "traffic": profiled_traffic("do_forward_backward"),
+                         "traffic_over_algorithmic": (
+                             profiled_traffic("do_forward_backward") / algorithmic_bytes(T, E, L)
+                             if profiled_traffic("do_forward_backward") else None),
                          "frac_of_nominal_8000_GBs": achieved / NOMINAL_HBM_GBS},
             "assignments_per_s": value * k,
             "split_entry_points": {"us": {k_: v * 1e3 for k_, v in stage_ms.items()},

@@ -373,37 +373,53 @@ loss_mma_kernel(const __grid_constant__ CUtensorMap zmap, const __grid_constant_
                     const unsigned char *zrow = sZ + (size_t)box_id(cc) * kBoxBytes + lane * 128;
                     const uint32_t tl = tl0 + 32 * cc;
 #pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-                        uint32_t hi[16], lo[16];
-                        tmem_ld16(tl + 16 * h, hi);
-                        tmem_ld16(tl + kE + 16 * h, lo);
-                        float z[16];
+                    for (int h = 0; h < 4; ++h) {
+                        uint32_t hi[8], lo[8];
+                        tmem_ld8(tl + 8 * h, hi);
+                        tmem_ld8(tl + kE + 8 * h, lo);
+                        float z[8];
 #pragma unroll
-                        for (int q = 0; q < 4; ++q) {
+                        for (int q = 0; q < 2; ++q) {
                             const float4 v = *reinterpret_cast<const float4 *>(
-                                zrow + (((4 * h + q) ^ (lane & 7)) << 4));
+                                zrow + (((2 * h + q) ^ (lane & 7)) << 4));
                             z[4 * q] = v.x;
                             z[4 * q + 1] = v.y;
                             z[4 * q + 2] = v.z;
                             z[4 * q + 3] = v.w;
                         }
                         tmem_wait_ld();
-                        // s = 1 / (1 + 2^(-z log2 e)): 0 when the power
-                        // overflows (z < -88), 1 when it underflows; the
-                        // Jacobian entry s (1 - s) as s - s^2 in one FMA (its
-                        // absolute error is an ulp of s, far below the
-                        // gradient's tolerance relative to its largest entry)
+                        // s = 1 / (1 + 2^(-z log2 e)), four at a time with one
+                        // reciprocal: with y_q = 1 + 2^(-z_q log2 e) and
+                        // r = 1 / (y0 y1 y2 y3), 1 / y0 = r y1 (y2 y3) and so
+                        // on (the exponent is capped at 30 so the product
+                        // stays finite: s >= 2^-30 below z = -20.8, an
+                        // absolute error under 1e-9).  The Jacobian entry
+                        // s (1 - s) is s - s^2 in one FMA (its absolute error
+                        // is an ulp of s, far below the gradient's tolerance
+                        // relative to its largest entry).
 #pragma unroll
-                        for (int e = 0; e < 16; ++e) {
-                            const float V = fmaf(__uint_as_float(hi[e]), 2048.0f, __uint_as_float(lo[e]));
-                            const float s = rcp_approx(1.0f + ex2_approx(z[e] * -kLog2e));
-                            S += s;
-                            SV = fmaf(s, V, SV);
-                            hi[e] = __float_as_uint(fmaf(-s, s, s));
-                            lo[e] = __float_as_uint(V);
+                        for (int g4 = 0; g4 < 2; ++g4) {
+                            float y[4];
+#pragma unroll
+                            for (int q = 0; q < 4; ++q)
+                                y[q] = 1.0f + ex2_approx(fminf(z[4 * g4 + q] * -kLog2e, 30.0f));
+                            const float p01 = y[0] * y[1], p23 = y[2] * y[3];
+                            const float r = rcp_approx(p01 * p23);
+                            const float r01 = r * p23, r23 = r * p01;
+                            const float sq4[4] = {r01 * y[1], r01 * y[0], r23 * y[3], r23 * y[2]};
+#pragma unroll
+                            for (int q = 0; q < 4; ++q) {
+                                const int e = 4 * g4 + q;
+                                const float V = fmaf(__uint_as_float(hi[e]), 2048.0f, __uint_as_float(lo[e]));
+                                const float s = sq4[q];
+                                S += s;
+                                SV = fmaf(s, V, SV);
+                                hi[e] = __float_as_uint(fmaf(-s, s, s));
+                                lo[e] = __float_as_uint(V);
+                            }
                         }
-                        tmem_st16(tl + 16 * h, hi);
-                        tmem_st16(tl + kE + 16 * h, lo);
+                        tmem_st8(tl + 8 * h, hi);
+                        tmem_st8(tl + kE + 8 * h, lo);
                     }
                 }
                 tmem_wait_st();
@@ -507,19 +523,19 @@ loss_mma_kernel(const __grid_constant__ CUtensorMap zmap, const __grid_constant_
                 unsigned char *zrow = sZ + (size_t)box_id(cc) * kBoxBytes + lane * 128;
                 const uint32_t tl = tl0 + 32 * cc;
 #pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    uint32_t jac[16], vv[16];
-                    tmem_ld16(tl + 16 * h, jac);
-                    tmem_ld16(tl + kE + 16 * h, vv);
+                for (int h = 0; h < 4; ++h) {
+                    uint32_t jac[8], vv[8];
+                    tmem_ld8(tl + 8 * h, jac);
+                    tmem_ld8(tl + kE + 8 * h, vv);
                     tmem_wait_ld();
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) {
+                    for (int q = 0; q < 2; ++q) {
                         float4 o;
                         o.x = __uint_as_float(jac[4 * q]) * fmaf(-cs, __uint_as_float(vv[4 * q]), csA);
                         o.y = __uint_as_float(jac[4 * q + 1]) * fmaf(-cs, __uint_as_float(vv[4 * q + 1]), csA);
                         o.z = __uint_as_float(jac[4 * q + 2]) * fmaf(-cs, __uint_as_float(vv[4 * q + 2]), csA);
                         o.w = __uint_as_float(jac[4 * q + 3]) * fmaf(-cs, __uint_as_float(vv[4 * q + 3]), csA);
-                        *reinterpret_cast<float4 *>(zrow + (((4 * h + q) ^ (lane & 7)) << 4)) = o;
+                        *reinterpret_cast<float4 *>(zrow + (((2 * h + q) ^ (lane & 7)) << 4)) = o;
                     }
                 }
             }
