@@ -228,6 +228,27 @@ def reduce_max(x: float, world: int, device) -> float:
     return float(t.item())
 
 
+def graph_ms_per_call(fn, reps: int) -> float:
+    """Device time of one call of fn(r): reps calls captured in one CUDA graph
+    (after one eager call that sets up any per-device state), the replay timed
+    with CUDA events on the launching stream."""
+    fn(0)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for r in range(reps):
+            fn(r)
+    g.replay()
+    torch.cuda.synchronize()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record()
+    g.replay()
+    b.record()
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / reps
+
+
 def replica_throughput(units_per_rank: float, seconds: float, world: int, device) -> tuple:
     """Whole-job rate of `world` independent replicas: the units of all ranks
     over the slowest rank's time.  Returns (rate, slowest seconds)."""
@@ -452,27 +473,26 @@ def run_ours(args, rank, world, local):
     if st != 0:
         raise RuntimeError(f"device status after the timed region: {dl.status_string(st)}")
 
-    # Per-stage durations: the same launches through the split entry points,
-    # with events between them on the launching stream.
-    stage_ms = {"signatures": 0.0, "pairwise_hamming": 0.0, "loss_fwd_bwd": 0.0}
+    # Per-stage durations through the split entry points: each stage's calls
+    # (reps of them over the rotating sets, inputs left by the stage before)
+    # captured in one CUDA graph, the replay timed with events, so that the
+    # host's launch overhead between calls is not counted as device time.
     reps = max(20, min(args.steps, 2000))
-    evs = [torch.cuda.Event(enable_timing=True) for _ in range(4 * reps)]
-    for r in range(reps):
-        z, out = sets[r % N_SETS]
-        e = evs[4 * r:4 * r + 4]
-        e[0].record(stream)
+    for r in range(N_SETS):
+        z, out = sets[r]
         dl.signatures(z, k, out.bits, out.counts)
-        e[1].record(stream)
         dl.pairwise_hamming(out.bits, T, out.D)
-        e[2].record(stream)
-        dl.loss_fwd_bwd(z, out.bits, out.D, k, w.gate, workspace=out.workspace, dlogits=out.dlogits)
-        e[3].record(stream)
     torch.cuda.synchronize()
-    for r in range(reps):
-        e = evs[4 * r:4 * r + 4]
-        stage_ms["signatures"] += e[0].elapsed_time(e[1]) / reps
-        stage_ms["pairwise_hamming"] += e[1].elapsed_time(e[2]) / reps
-        stage_ms["loss_fwd_bwd"] += e[2].elapsed_time(e[3]) / reps
+    stage_calls = {
+        "signatures": lambda r: dl.signatures(sets[r % N_SETS][0], k, sets[r % N_SETS][1].bits,
+                                              sets[r % N_SETS][1].counts),
+        "pairwise_hamming": lambda r: dl.pairwise_hamming(sets[r % N_SETS][1].bits, T,
+                                                          sets[r % N_SETS][1].D),
+        "loss_fwd_bwd": lambda r: dl.loss_fwd_bwd(
+            sets[r % N_SETS][0], sets[r % N_SETS][1].bits, sets[r % N_SETS][1].D, k, w.gate,
+            workspace=sets[r % N_SETS][1].workspace, dlogits=sets[r % N_SETS][1].dlogits),
+    }
+    stage_ms = {name: graph_ms_per_call(fn, reps) for name, fn in stage_calls.items()}
     # Routing outputs (Sec. 3.1.1): do_routing alone, and the DO-loss step that
     # also writes them from the same selection pass.
     routes = [dl.Routing(L, T, E, k, dev) for _ in range(N_SETS)]

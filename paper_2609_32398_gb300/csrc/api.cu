@@ -145,7 +145,7 @@ do_status do_pairwise_hamming_accumulate(const uint32_t *bits, int64_t T, int32_
     if (st != DO_OK) return st;
     if (!bits || !D) return DO_ERR_INVALID_ARG;
     if (!aligned(bits, 4) || !aligned(D, 4)) return DO_ERR_INVALID_ARG;
-    return from_cuda(dol::launch_hamming_accumulate(bits, p, D, nullptr, (cudaStream_t)stream));
+    return from_cuda(dol::launch_hamming_accumulate(bits, p, D, (cudaStream_t)stream));
 }
 
 do_status do_offdiag_variance(const int64_t *origin_do, int64_t T, int32_t E, int32_t k, int32_t L,

@@ -95,8 +95,7 @@ cudaError_t launch_signatures(const float *logits, const Problem &p, uint32_t *b
                               const RouteOut &route = RouteOut{nullptr, nullptr, 0});
 cudaError_t launch_hamming(const uint32_t *bits, const Problem &p, int *D, cudaStream_t s);
 cudaError_t launch_add_distances(const int *D, int *D_sum, int64_t n, cudaStream_t s);
-cudaError_t launch_hamming_accumulate(const uint32_t *bits, const Problem &p, int *D, int *counts,
-                                      cudaStream_t s);
+cudaError_t launch_hamming_accumulate(const uint32_t *bits, const Problem &p, int *D, cudaStream_t s);
 cudaError_t launch_origin_do(const int *D, const Problem &p, long long *origin_do, cudaStream_t s);
 // var [L] (fp64) = the variance of the off-diagonal entries of each problem's
 // local Hamming matrix from its origin_do (App. C.1).

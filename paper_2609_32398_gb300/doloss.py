@@ -147,15 +147,17 @@ def signatures(logits: torch.Tensor, k: int, bits=None, counts=None):
     return bits, counts
 
 
-def pairwise_hamming(bits: torch.Tensor, T: int, D=None):
-    """Step 2: D [L,E,E] int32 from bits [L,E,W]."""
+def pairwise_hamming(bits: torch.Tensor, T: int, D=None, accumulate=False):
+    """Step 2: D [L,E,E] int32 from bits [L,E,W]; with accumulate, D += it."""
     if bits.dim() == 2:
         bits = bits.unsqueeze(0)
     L, E, _ = bits.shape
     if D is None:
+        if accumulate:
+            raise ValueError("accumulate needs the D to add to")
         D = torch.empty(L, E, E, dtype=torch.int32, device=bits.device)
-    _check("do_pairwise_hamming", lib().do_pairwise_hamming(bits.data_ptr(), T, E, L, D.data_ptr(),
-                                                            _stream(bits)))
+    name = "do_pairwise_hamming_accumulate" if accumulate else "do_pairwise_hamming"
+    _check(name, getattr(lib(), name)(bits.data_ptr(), T, E, L, D.data_ptr(), _stream(bits)))
     return D
 
 

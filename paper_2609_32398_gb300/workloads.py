@@ -24,6 +24,7 @@ from __future__ import annotations
 
 from dataclasses import dataclass, replace
 
+import numpy as np
 import torch
 
 GATE_SIGMOID_NORM = 0
@@ -125,6 +126,21 @@ def random_logits(T: int, E: int, L: int = 1, seed: int = 0, device="cpu",
     if ties:
         z = torch.round(z * 2.0) / 2.0
     return z
+
+
+def random_signatures(T: int, E: int, L: int = 1, seed: int = 0, density_log2: int = 1):
+    """Load signatures [L, E, W] uint32 (numpy) for the pairwise-distance sweeps:
+    each bit is 1 with probability 2^-density_log2 (the AND of that many
+    uniform words; 4 gives k/E = 8/128), token t of an expert at bit t % 32 of
+    word t // 32, and the bits past T in the last word zero."""
+    W = (T + 31) // 32
+    g = np.random.default_rng(seed)
+    bits = np.full((L, E, W), 0xFFFFFFFF, np.uint32)
+    for _ in range(max(1, density_log2)):
+        bits &= g.integers(0, 1 << 32, size=(L, E, W), dtype=np.uint64).astype(np.uint32)
+    if T % 32:
+        bits[..., W - 1] &= np.uint32((1 << (T % 32)) - 1)
+    return bits
 
 
 def router_inputs(T: int, H: int, E: int = 128, L: int = 1, seed: int = 0, device="cpu"):

@@ -406,3 +406,19 @@ def test_dense_p_reading_against_the_renormalized_one():
     C1 = oracle.direction_mode(z, f, mode=1)
     assert C1.sum() == pytest.approx(T * (E - k), rel=1e-12)
 
+
+
+def test_random_signatures_are_packed_selections():
+    """The sweep generator's words unpack to a 0/1 matrix that the oracle packs
+    back to the same words (bits past T zero), with about the asked density,
+    and the oracle's word-wise distances equal its token-wise ones on them."""
+    T, E, L = 1000 + 13, 9, 2
+    bits = workloads.random_signatures(T, E, L, seed=4, density_log2=3)
+    for l in range(L):
+        f = np.zeros((T, E), np.uint8)
+        for i in range(E):
+            for t in range(T):
+                f[t, i] = (int(bits[l, i, t // 32]) >> (t % 32)) & 1
+        assert np.array_equal(oracle.pack(f), bits[l])
+        assert abs(f.mean() - 1 / 8) < 0.02
+        assert np.array_equal(oracle.hamming_bits(bits[l], T), oracle.hamming(f))
