@@ -232,6 +232,8 @@ def graph_ms_per_call(fn, reps: int) -> float:
     """Device time of one call of fn(r): reps calls captured in one CUDA graph
     (after one eager call that sets up any per-device state), the replay timed
     with CUDA events on the launching stream."""
+    import torch
+
     fn(0)
     torch.cuda.synchronize()
     g = torch.cuda.CUDAGraph()
@@ -454,18 +456,43 @@ def run_ours(args, rank, world, local):
             torch.cuda.synchronize()
     torch.cuda.synchronize()
 
+    # The K timed steps are captured in one CUDA graph (the calls a training
+    # step makes, with the host's per-launch cost out of the device timeline)
+    # and replayed once untimed before the timed replay.
+    timing = "cuda_graph"
+    g_steps = torch.cuda.CUDAGraph()
+    try:
+        with torch.cuda.graph(g_steps):
+            for i in range(args.steps):
+                step(i)
+        g_steps.replay()
+        torch.cuda.synchronize()
+    except RuntimeError as ex:
+        g_steps = None
+        timing = f"eager loop (graph capture failed: {str(ex)[:80]})"
+        torch.cuda.synchronize()
     barrier(world)
     torch.cuda.synchronize()
     ev0 = torch.cuda.Event(enable_timing=True)
     ev1 = torch.cuda.Event(enable_timing=True)
     ev0.record(stream)
-    for i in range(args.steps):
-        step(i)
+    if g_steps is not None:
+        g_steps.replay()
+    else:
+        for i in range(args.steps):
+            step(i)
     ev1.record(stream)
     torch.cuda.synchronize()
     barrier(world)
     clocks = sampler.stop()
     ms = ev0.elapsed_time(ev1)
+    # the same steps as a Python loop of calls, for comparison
+    ev0.record(stream)
+    for i in range(args.steps):
+        step(i)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    eager_ms = ev0.elapsed_time(ev1) / args.steps
     value, seconds = replica_throughput(T * L * args.steps, ms * 1e-3, world, dev)
     ms_per_step = seconds * 1e3 / args.steps
 
@@ -502,15 +529,10 @@ def run_ours(args, rank, world, local):
                                    route=routes[r % N_SETS])
     torch.cuda.synchronize()
 
+    # Device time per call: reps calls in one CUDA graph (a Python loop of
+    # several launches per call is limited by the host's launch rate).
     def time_calls(fn):
-        a = torch.cuda.Event(enable_timing=True)
-        b = torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        for r in range(reps):
-            fn(r)
-        b.record(stream)
-        torch.cuda.synchronize()
-        return a.elapsed_time(b) / reps
+        return graph_ms_per_call(fn, reps)
 
     route_ms = time_calls(lambda r: dl.routing(sets[r % N_SETS][0], k, w.gate, out=routes[r % N_SETS]))
     routed_ms = time_calls(lambda r: dl.forward_backward_routed(
@@ -599,7 +621,7 @@ def run_ours(args, rank, world, local):
     def maxvio_call(cnt, er, E_, L_):
         # the C entry point with preallocated outputs: launches back to back
         st_ = lib.do_maxvio(cnt.data_ptr(), er.data_ptr(), E_, R_ep, L_, None, mv_out.data_ptr(),
-                            None, stream.cuda_stream)
+                            None, torch.cuda.current_stream().cuda_stream)
         if st_ != 0:
             raise RuntimeError(dl.status_string(st_))
     mv1_ms = time_calls(lambda r: maxvio_call(c1, er1, E, L))
@@ -765,6 +787,10 @@ def run_ours(args, rank, world, local):
                              if profiled_traffic("do_forward_backward") else None),
                          "frac_of_nominal_8000_GBs": achieved / NOMINAL_HBM_GBS},
             "assignments_per_s": value * k,
+            "timing": timing,
+            "eager_loop": {"what": "the same steps as a Python loop of do_forward_backward calls",
+                           "us_per_step": eager_ms * 1e3,
+                           "tokens_per_s": T * L / (eager_ms * 1e-3)},
             "split_entry_points": {"us": {k_: v * 1e3 for k_, v in stage_ms.items()},
                                    "GB/s": split_gbs},
             "size_matched_copy": {

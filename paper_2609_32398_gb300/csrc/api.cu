@@ -459,6 +459,29 @@ do_status do_routed_backward(const float *logits, int64_t T, int32_t E, int32_t 
     // summed over ranks or micro-batches (Eq. global_do), read as given.
     const bool local = d_scale == 1.0f;
     cudaError_t e;
+    if (!local && split_fast(p, logits, bits, D) && aligned(dlogits, 16) &&
+        dol::loss_mma_supported(p, gate, logits, D, dlogits, true) &&
+        (!rg || (aligned(expert_ids, 16) && aligned(grad_combine, 16)))) {
+        // a given matrix: its image of D' is built here, with a flag per
+        // problem saying whether the two fp16 pieces hold it exactly; the
+        // tensor-core kernel takes the exact problems (routing gradient in its
+        // epilogue), the ALU kernel and the routing-gradient kernel the others
+        unsigned char *bimg = reinterpret_cast<unsigned char *>(ws + w.bimg);
+        int *img_ok = reinterpret_cast<int *>(ws + w.img_ok);
+        e = dol::launch_dprime_image(D, p, bimg, img_ok, s);
+        if (e == cudaSuccess)
+            e = dol::launch_loss_mma(logits, idx, bimg, nullptr, p, d_scale, grad_scale, loss,
+                                     dlogits, partials, done, status, nullptr, s, expert_ids,
+                                     grad_combine, img_ok);
+        if (e == cudaSuccess)
+            e = dol::launch_loss_fast(logits, idx, D, nullptr, nullptr, p, gate, d_scale,
+                                      grad_scale, loss, nullptr, dlogits, partials, done, status,
+                                      nullptr, s, img_ok);
+        if (e == cudaSuccess && rg)
+            e = dol::launch_route_backward(logits, expert_ids, grad_combine, p.T * p.L, E, k, gate,
+                                           1, dlogits, status, s, img_ok, p.T);
+        return from_cuda(e);
+    }
     if (split_fast(p, logits, bits, D) && aligned(dlogits, 16)) {
         if (local && split_mma(p, gate, logits, D) &&
             dol::loss_mma_supported(p, gate, logits, D, dlogits) &&

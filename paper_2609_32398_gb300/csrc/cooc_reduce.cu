@@ -110,6 +110,66 @@ cudaError_t run_reduce(const uint32_t *partials, int P1, const int *n_acc, const
                               origin_do, r_base, r_mult);
 }
 
+// The image of D' from a given matrix D (a matrix summed over ranks or
+// micro-batches, Eq. global_do): off the diagonal D_ab, on it -R_a with R_a =
+// sum_{b != a} D_ab (D symmetric).  img_ok[layer] = 1 when the two fp16
+// pieces are exact for this matrix (0 <= D_ab < 2^22 off the diagonal,
+// D_aa = 0, R_a < 2^23), else 0: the tensor-core loss kernel takes the
+// problems with 1, the ALU kernel the others.  One CTA per problem; a thread
+// builds one 16-byte chunk of row n of each piece (8 consecutive k = a) from
+// D[n][a .. a + 7], the 16 threads of row n (a half warp) add R_n with
+// shuffles, and the chunks are written whole (the 128-byte swizzle moves
+// whole 16-byte chunks).
+__global__ void __launch_bounds__(kRedThreads)
+dprime_image_kernel(const int *__restrict__ D, unsigned char *__restrict__ bimg,
+                    int *__restrict__ img_ok) {
+    constexpr int E = 128;
+    const int layer = blockIdx.x;
+    const int *Dl = D + (size_t)layer * E * E;
+    unsigned char *img = bimg + (size_t)layer * kBImageBytes;
+    pdl_wait();
+    pdl_trigger();
+    int ok = 1;
+#pragma unroll
+    for (int pass = 0; pass < 2; ++pass) {
+        const int item = pass * kRedThreads + (int)threadIdx.x;
+        const int n = item >> 4, a0 = 8 * (item & 15);
+        const int4 v0 = __ldg(reinterpret_cast<const int4 *>(Dl + n * E + a0));
+        const int4 v1 = __ldg(reinterpret_cast<const int4 *>(Dl + n * E + a0 + 4));
+        const int v[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+        long long row = 0;
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            if (a0 + u == n) {
+                ok &= v[u] == 0;
+            } else {
+                ok &= v[u] >= 0 && v[u] < (1 << 22);
+                row += v[u];
+            }
+        }
+#pragma unroll
+        for (int o = 8; o > 0; o >>= 1) row += __shfl_xor_sync(kFull, row, o);
+        ok &= row < (1 << 23);
+        uint32_t hw[4], lw[4];
+#pragma unroll
+        for (int u = 0; u < 8; u += 2) {
+            int h0, l0, h1, l1;
+            dprime_pieces(a0 + u == n, a0 + u == n ? (int)row : v[u], &h0, &l0);
+            dprime_pieces(a0 + u + 1 == n, a0 + u + 1 == n ? (int)row : v[u + 1], &h1, &l1);
+            hw[u / 2] = (uint32_t)__half_as_ushort(__int2half_rn(h0)) |
+                        ((uint32_t)__half_as_ushort(__int2half_rn(h1)) << 16);
+            lw[u / 2] = (uint32_t)__half_as_ushort(__int2half_rn(l0)) |
+                        ((uint32_t)__half_as_ushort(__int2half_rn(l1)) << 16);
+        }
+        *reinterpret_cast<uint4 *>(img + sw128_k16_offset(n, a0, 256)) =
+            make_uint4(hw[0], hw[1], hw[2], hw[3]);
+        *reinterpret_cast<uint4 *>(img + sw128_k16_offset(128 + n, a0, 256)) =
+            make_uint4(lw[0], lw[1], lw[2], lw[3]);
+    }
+    ok = __syncthreads_and(ok);
+    if (threadIdx.x == 0) img_ok[layer] = ok;
+}
+
 }  // namespace
 
 cudaError_t launch_cooc_reduce(const uint32_t *partials, int P1, const int *n_acc, const Problem &p,
@@ -119,6 +179,21 @@ cudaError_t launch_cooc_reduce(const uint32_t *partials, int P1, const int *n_ac
     if (p.E == 64) return run_reduce<64>(partials, P1, n_acc, p, D, counts, nullptr, origin_do, s);
     if (p.E == 128) return run_reduce<128>(partials, P1, n_acc, p, D, counts, bimg, origin_do, s);
     return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_dprime_image(const int *D, const Problem &p, unsigned char *bimg, int *img_ok,
+                                cudaStream_t s) {
+    if (p.E != 128) return cudaErrorInvalidValue;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)p.L);
+    cfg.blockDim = dim3(kRedThreads);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, dprime_image_kernel, D, bimg, img_ok);
 }
 
 }  // namespace dol

@@ -71,9 +71,10 @@ struct ZeroSpans {
 //   n_acc           [L][E] int32, counts summed by the signatures CTAs (kept at
 //                   zero between calls: the loss kernel clears it after use)
 //   bimg            [L][kBImageBytes], the fp16 image of D' (E = 128 only)
+//   img_ok          [L] int32, 1 where the image of a given (summed) D is exact
 //   route_base      route_scratch_ints int32, scratch of the dispatch order
 struct WsLayout {
-    size_t done, partials, idx, cooc_parts, n_acc, bimg, route_base, total;
+    size_t done, partials, idx, cooc_parts, n_acc, bimg, img_ok, route_base, total;
     int max_parts;  // partial slots per problem
 };
 // Signatures CTAs per problem on the fast path: min(SMs, kMaxSigCtas) / L.
@@ -123,10 +124,13 @@ cudaError_t launch_signatures_fast_routed(const float *logits, const Problem &p,
 int64_t route_chunks(const Problem &p);
 int64_t route_scratch_ints(const Problem &p);
 // Backward of the combine weights to the logits over `rows` token rows
-// (route_bwd.cu); status bit 2 for an id outside [0, E).
+// (route_bwd.cu); status bit 2 for an id outside [0, E).  skip (with
+// accumulate only; may be null): [rows / layer_rows] flags, the rows of a
+// problem whose flag is nonzero are left alone.
 cudaError_t launch_route_backward(const float *z, const int32_t *ids, const float *g, int64_t rows,
                                   int32_t E, int32_t k, int32_t gate, int32_t accumulate,
-                                  float *dz, int32_t *status_flags, cudaStream_t s);
+                                  float *dz, int32_t *status_flags, cudaStream_t s,
+                                  const int *skip = nullptr, int64_t layer_rows = 0);
 
 // n_zero (may be null): an [L][E] accumulator cleared once the kernels before
 // these have finished (the scan kernel does it after its dependency wait).
@@ -153,7 +157,7 @@ cudaError_t launch_idx_from_bits(const uint32_t *bits, const Problem &p, uint8_t
 // column sum of D.
 // Tensor-core loss path (E = 128, sigmoid-norm gate, k in {1,2,4,8}, T <= 2^22).
 bool loss_mma_supported(const Problem &p, int gate, const float *logits, const int *D,
-                        const float *dlogits);
+                        const float *dlogits, bool image_checked = false);
 int loss_mma_ctas_per_problem(const Problem &p);
 // bimg: the fp16 image of D' written by launch_cooc_reduce for these tokens
 // (which also gives origin_do on this path).
@@ -161,12 +165,12 @@ cudaError_t launch_loss_mma(const float *logits, const uint8_t *idx, const unsig
                             int *n_zero, const Problem &p, float d_scale, float grad_scale,
                             float *loss, float *dlogits, double *partials, int *done, int *status,
                             int *status_out, cudaStream_t s, const int *rg_ids = nullptr,
-                            const float *rg_g = nullptr);
+                            const float *rg_g = nullptr, const int *img_ok = nullptr);
 cudaError_t launch_loss_fast(const float *logits, const uint8_t *idx, const int *D,
                              const int *counts, int *n_zero, const Problem &p, int gate,
                              float d_scale, float grad_scale, float *loss, long long *origin_do,
                              float *dlogits, double *partials, int *done, int *status,
-                             int *status_out, cudaStream_t s);
+                             int *status_out, cudaStream_t s, const int *img_ok = nullptr);
 
 // Co-occurrence counts c_ab (a <= b) of one CTA are kept as a triangle whose
 // row a holds columns (a & ~3) .. E-1, so that every row starts 16-byte
@@ -216,6 +220,10 @@ size_t cooc_partial_words(int E);
 cudaError_t launch_cooc_reduce(const uint32_t *partials, int P1, const int *n_acc, const Problem &p,
                                int *D, int *counts, unsigned char *bimg, long long *origin_do,
                                cudaStream_t s);
+// The image of D' from a given [L][128][128] matrix D (summed over ranks or
+// micro-batches), and img_ok [L] = 1 where its two fp16 pieces are exact.
+cudaError_t launch_dprime_image(const int *D, const Problem &p, unsigned char *bimg, int *img_ok,
+                                cudaStream_t s);
 
 // ---------------------------------------------------------------- device helpers
 

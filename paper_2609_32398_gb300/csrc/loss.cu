@@ -272,7 +272,8 @@ WsLayout ws_layout(const Problem &p) {
     w.bimg = up(w.n_acc + ((fast_k && fast_e) ? sizeof(int) * (size_t)p.L * p.E : 0));
     // the dispatch order of a routed call may run beside the loss kernel: its
     // scratch has a region of its own
-    w.route_base = up(w.bimg + ((fast_k && p.E == 128) ? (size_t)kBImageBytes * (size_t)p.L : 0));
+    w.img_ok = up(w.bimg + ((fast_k && p.E == 128) ? (size_t)kBImageBytes * (size_t)p.L : 0));
+    w.route_base = up(w.img_ok + ((fast_k && p.E == 128) ? sizeof(int) * (size_t)p.L : 0));
     w.total = up(w.route_base + sizeof(int) * (size_t)route_scratch_ints(p));
     return w;
 }

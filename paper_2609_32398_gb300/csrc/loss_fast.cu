@@ -93,6 +93,9 @@ struct LossArgs {
     long long *origin_do;
     int *status;
     int *status_out;  // may be null: the last CTA ORs the status word into it
+    // layers whose img_ok flag is 1 went to the tensor-core kernel: skipped
+    // here (may be null)
+    const int *img_ok;
 };
 
 template <int E, int K, int kGate, bool kRFromCounts>
@@ -138,6 +141,7 @@ loss_fast_kernel(const LossArgs a) {
     }
     __syncthreads();
     pdl_wait();  // D, idx and the cleared counters come from the previous kernels
+    if (a.img_ok && __ldg(a.img_ok + layer) != 0) return;
     if (threadIdx.x == 0) {
         mbar_arrive_expect_tx(&bar, (uint32_t)(sizeof(int) * E * E));
         bulk_load(sD, a.D + (int64_t)layer * E * E, (uint32_t)(sizeof(int) * E * E), &bar);
@@ -464,7 +468,7 @@ cudaError_t launch_loss_fast(const float *logits, const uint8_t *idx, const int 
                              const int *counts, int *n_zero, const Problem &p, int gate,
                              float d_scale, float grad_scale, float *loss, long long *origin_do,
                              float *dlogits, double *partials, int *done, int *status,
-                             int *status_out, cudaStream_t s) {
+                             int *status_out, cudaStream_t s, const int *img_ok) {
     int P = 1, tpc = 32;
     loss_fast_grid(p, &P, &tpc);
     const double norm = 1.0 / ((double)p.T * (double)p.T * (double)p.k);
@@ -486,6 +490,7 @@ cudaError_t launch_loss_fast(const float *logits, const uint8_t *idx, const int 
     args.origin_do = origin_do;
     args.status = status;
     args.status_out = status_out;
+    args.img_ok = img_ok;
     if (counts) {
         if (p.E == 32) return dispatch_loss_k<32, true>(args, gate, P, p, s);
         if (p.E == 64) return dispatch_loss_k<64, true>(args, gate, P, p, s);

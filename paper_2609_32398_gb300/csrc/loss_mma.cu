@@ -132,6 +132,9 @@ struct MmaArgs {
     // gradient of their combine weights [L][T][K]
     const int *rg_ids;
     const float *rg_g;
+    // a matrix summed over ranks (Eq. global_do): img_ok [L] from the image
+    // kernel; a layer whose flag is 0 is left to the ALU kernel (may be null)
+    const int *img_ok;
 };
 
 // K ints and K floats of one token row (16-, 8- or 4-byte loads)
@@ -247,6 +250,20 @@ loss_mma_kernel(const __grid_constant__ CUtensorMap zmap, const __grid_constant_
     }
 
     pdl_wait();  // the image of D', D and the selected experts come from the previous kernels
+    if (a.img_ok && __ldg(a.img_ok + layer) == 0) {
+        // this problem's matrix does not fit the image (the ALU kernel that
+        // follows takes it): wait for the logits requested above, release
+        // TMEM and leave
+        if (epi && lane == 0 && z_issued) {
+            mbar_wait(&zfull[box_id(0)], 0u, a.status);
+            mbar_wait(&zfull[box_id(1)], 0u, a.status);
+        }
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+        if (warp == 0) tmem_dealloc(tmem, kTmemCols);
+        return;
+    }
 
     float tok_sum = 0.0f;  // sum of A_t over this thread's tokens (at most a few tiles)
     if (warp == 0) {
@@ -649,11 +666,12 @@ cudaError_t run_mma(const CUtensorMap &zmap, const CUtensorMap &dzmap, const Mma
 }  // namespace
 
 bool loss_mma_supported(const Problem &p, int gate, const float *logits, const int *D,
-                        const float *dlogits) {
+                        const float *dlogits, bool image_checked) {
     const bool k_ok = p.k == 1 || p.k == 2 || p.k == 4 || p.k == 8;
     auto al = [](const void *q) { return reinterpret_cast<uintptr_t>(q) % 16 == 0; };
     // R_i <= (E - 1) T must stay below 2^23 for the two-piece split of D'
-    const bool t_ok = (int64_t)(kE - 1) * p.T < (int64_t)(1 << 23);
+    // (unless the image kernel checks the split of a given matrix)
+    const bool t_ok = image_checked || (int64_t)(kE - 1) * p.T < (int64_t)(1 << 23);
     return p.E == kE && gate == 0 && k_ok && dlogits != nullptr && t_ok && al(logits) &&
            al(dlogits) && al(D);
 }
@@ -670,7 +688,8 @@ int loss_mma_ctas_per_problem(const Problem &p) {
 cudaError_t launch_loss_mma(const float *logits, const uint8_t *idx, const unsigned char *bimg, int *n_zero, const Problem &p, float d_scale,
                             float grad_scale, float *loss, float *dlogits,
                             double *partials, int *done, int *status, int *status_out,
-                            cudaStream_t s, const int *rg_ids, const float *rg_g) {
+                            cudaStream_t s, const int *rg_ids, const float *rg_g,
+                            const int *img_ok) {
     if (!bimg) return cudaErrorInvalidValue;
     CUtensorMap zmap, dzmap;
     if (!encode_tensor_map_3d_f32(&zmap, logits, (uint64_t)p.L, (uint64_t)p.T, (uint64_t)kE, 32) ||
@@ -695,6 +714,7 @@ cudaError_t launch_loss_mma(const float *logits, const uint8_t *idx, const unsig
     args.status_out = status_out;
     args.rg_ids = rg_ids;
     args.rg_g = rg_g;
+    args.img_ok = img_ok;
     if (rg_ids && rg_g) {
         switch (p.k) {
             case 1: return run_mma<1, true>(zmap, dzmap, args, gx, p.L, s);

@@ -44,12 +44,14 @@ __device__ __forceinline__ float group_max(float v, int G) {
 // accumulate = 0: the rows are overwritten (zeros, then the chosen entries);
 // accumulate = 1: the chosen entries are added in place (RED.ADD; one
 // contribution per entry when the ids of a row are distinct, hence the same
-// sum every run).
+// sum every run).  skip (accumulate only, may be null): rows r of problems
+// r / layer_rows whose flag is nonzero are left alone (their gradient was
+// added by the tensor-core loss kernel).
 __global__ void __launch_bounds__(kThreads)
 route_backward_kernel(const float *__restrict__ z, const int32_t *__restrict__ ids,
                       const float *__restrict__ g, int64_t rows, int32_t E, int32_t k, int32_t G,
                       int32_t gate, int32_t accumulate, float *__restrict__ dz,
-                      int32_t *status_flags) {
+                      int32_t *status_flags, const int *__restrict__ skip, int64_t layer_rows) {
     const int lane = threadIdx.x & 31;
     const int per_pass = 32 / G;
     const int j = lane & (G - 1);
@@ -59,7 +61,7 @@ route_backward_kernel(const float *__restrict__ z, const int32_t *__restrict__ i
     int bad = 0;
     for (int64_t base = warp * per_pass; base < rows; base += nwarps * per_pass) {
         const int64_t r = base + lane / G;
-        const bool live = r < rows;
+        const bool live = r < rows && !(skip && __ldg(skip + r / layer_rows) != 0);
         const float *zr = z + (live ? r : 0) * (int64_t)E;
         const int32_t *ir = ids + (live ? r : 0) * (int64_t)k;
         const float *gr = g + (live ? r : 0) * (int64_t)k;
@@ -124,7 +126,7 @@ __global__ void __launch_bounds__(kThreads)
 route_backward_small_k(const float *__restrict__ z, const int32_t *__restrict__ ids,
                        const float *__restrict__ g, int64_t rows, int32_t E, int32_t k,
                        int32_t G, int32_t gate, int32_t accumulate, float *__restrict__ dz,
-                       int32_t *status_flags) {
+                       int32_t *status_flags, const int *__restrict__ skip, int64_t layer_rows) {
     const int lane = threadIdx.x & 31;
     const int per_pass = 32 / G;
     const int j = lane & (G - 1);
@@ -142,7 +144,7 @@ route_backward_small_k(const float *__restrict__ z, const int32_t *__restrict__ 
 #pragma unroll
         for (int u = 0; u < kU; ++u) {
             const int64_t r = base + (int64_t)u * per_pass + grp;
-            const bool on = has_q && r < rows;
+            const bool on = has_q && r < rows && !(skip && __ldg(skip + r / layer_rows) != 0);
             present |= on ? 1u << u : 0u;
             e[u] = on ? __ldg(ids + r * k + j) : 0;
             gq[u] = on ? __ldg(g + r * k + j) : 0.0f;
@@ -225,8 +227,10 @@ cudaError_t grid_for(size_t smem, int64_t warps, int *blocks) {
 
 cudaError_t launch_route_backward(const float *z, const int32_t *ids, const float *g, int64_t rows,
                                   int32_t E, int32_t k, int32_t gate, int32_t accumulate,
-                                  float *dz, int32_t *status_flags, cudaStream_t s) {
+                                  float *dz, int32_t *status_flags, cudaStream_t s,
+                                  const int *skip, int64_t layer_rows) {
     constexpr int kU = 4;
+    if (skip && (!accumulate || layer_rows < 1)) return cudaErrorInvalidValue;
     int G = 1;
     while (G < k && G < 32) G <<= 1;
     const int64_t per_warp = (k <= 32 ? kU : 1) * (int64_t)(32 / G);
@@ -236,11 +240,12 @@ cudaError_t launch_route_backward(const float *z, const int32_t *ids, const floa
                             : grid_for<route_backward_kernel>(0, warps, &blocks);
     if (e != cudaSuccess) return e;
     if (k <= 32)
-        route_backward_small_k<kU><<<blocks, kThreads, 0, s>>>(z, ids, g, rows, E, k, G, gate,
-                                                               accumulate, dz, status_flags);
+        route_backward_small_k<kU><<<blocks, kThreads, 0, s>>>(
+            z, ids, g, rows, E, k, G, gate, accumulate, dz, status_flags, skip, layer_rows);
     else
         route_backward_kernel<<<blocks, kThreads, 0, s>>>(z, ids, g, rows, E, k, G, gate,
-                                                          accumulate, dz, status_flags);
+                                                          accumulate, dz, status_flags, skip,
+                                                          layer_rows);
     return cudaGetLastError();
 }
 

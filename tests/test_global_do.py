@@ -201,3 +201,47 @@ def test_window_of_one_micro_batch_is_the_local_step():
     torch.cuda.synchronize()
     assert torch.equal(D, ref.D)
     assert torch.equal(losses[0], ref.loss) and torch.equal(grads[0], ref.dlogits)
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("with_route", [False, True])
+def test_summed_matrix_beyond_the_fp16_image_takes_the_alu_kernel(with_route):
+    """Eq. global_do with a given matrix at E = 128, two problems in one call:
+    problem 0's matrix (three local matrices' sum) fits the two fp16 pieces of
+    the tensor-core kernel's image of D', problem 1's (a 256-fold sum, row sums
+    above 2^23) does not and goes to the ALU kernel.  Both problems' loss and
+    gradient equal the oracle's for their matrix, with d_scale = 1/3, with and
+    without the combine weights' gradient added in the same call."""
+    import oracle
+    import paper_2609_32398_gb300.doloss as dl
+    from paper_2609_32398_gb300 import workloads
+
+    k, E, T, L = 8, 128, 4096 + 64, 2
+    z = workloads.random_logits(T, E, L=L, seed=321)
+    zc = z.cuda()
+    out, route = dl.routed_forward(zc, k, 0, with_routing=with_route)
+    torch.cuda.synchronize()
+    D_loc = [oracle.hamming(oracle.select(z[l].numpy(), k)) for l in range(L)]
+    mult = (3, 256)
+    D_sum = np.stack([D_loc[l].astype(np.int64) * mult[l] for l in range(L)])
+    assert D_sum[1].sum(axis=1).max() >= 1 << 23 > D_sum[0].sum(axis=1).max()
+    Dg = torch.from_numpy(D_sum.astype(np.int32)).cuda()
+    gq = None
+    if with_route:
+        gq = torch.randn(L, T, k, generator=torch.Generator().manual_seed(9)).cuda()
+    dl.routed_backward(zc, route.expert_ids if with_route else None, gq, k, 0, 1.5, out=out, D=Dg,
+                       d_scale=1.0 / 3)
+    torch.cuda.synchronize()
+    for l in range(L):
+        zl = z[l].numpy()
+        f = oracle.select(zl, k)
+        want = oracle.loss(D_sum[l], oracle.direction(zl, f), T, k, d_scale=1.0 / 3)
+        assert abs(float(out.loss[l]) - want) <= 1e-5 * abs(want), l
+        g = oracle.gate_backward(zl, oracle.dloss_dp(D_sum[l], f, T, k, d_scale=1.0 / 3),
+                                 grad_scale=1.5)
+        if with_route:
+            g = g + oracle.route_backward(zl, route.expert_ids[l].cpu().numpy(),
+                                          gq[l].double().cpu().numpy())
+        err = np.abs(out.dlogits[l].double().cpu().numpy() - g).max() / np.abs(g).max()
+        assert err <= 1e-4, (l, err)
+    assert dl.device_status(out.workspace) == 0
