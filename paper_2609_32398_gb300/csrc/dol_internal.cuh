@@ -95,6 +95,11 @@ cudaError_t launch_signatures(const float *logits, const Problem &p, uint32_t *b
                               int *counts, cudaStream_t s,
                               const RouteOut &route = RouteOut{nullptr, nullptr, 0});
 cudaError_t launch_hamming(const uint32_t *bits, const Problem &p, int *D, cudaStream_t s);
+// The fast selection at E = 256 (k in {1, 2, 4, 8}, 16-byte aligned logits):
+// signatures and counts (counts zero on entry), no co-occurrence.
+bool signatures_fast256_supported(const float *logits, const Problem &p);
+cudaError_t launch_signatures_fast256(const float *logits, const Problem &p, uint32_t *bits,
+                                      int *counts, cudaStream_t s);
 cudaError_t launch_add_distances(const int *D, int *D_sum, int64_t n, cudaStream_t s);
 cudaError_t launch_hamming_accumulate(const uint32_t *bits, const Problem &p, int *D, cudaStream_t s);
 cudaError_t launch_origin_do(const int *D, const Problem &p, long long *origin_do, cudaStream_t s);

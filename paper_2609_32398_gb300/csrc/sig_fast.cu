@@ -46,4 +46,21 @@ cudaError_t launch_signatures_fast(const float *logits, const Problem &p, uint32
     return dispatch_mode<128, false>(map, p, bits, counts, idx, cooc, zero, status, none, s);
 }
 
+bool signatures_fast256_supported(const float *logits, const Problem &p) {
+    const bool k_ok = p.k == 1 || p.k == 2 || p.k == 4 || p.k == 8;
+    return p.E == 256 && k_ok && (reinterpret_cast<uintptr_t>(logits) % 16 == 0) &&
+           (int64_t)p.L * p.T + 32 < (int64_t)INT_MAX;
+}
+
+cudaError_t launch_signatures_fast256(const float *logits, const Problem &p, uint32_t *bits,
+                                      int *counts, cudaStream_t s) {
+    CUtensorMap map;
+    if (!encode_tensor_map_2d_f32(&map, logits, (uint64_t)p.L * p.T, (uint64_t)p.E, 32))
+        return cudaErrorInvalidValue;
+    const RouteOut none = {nullptr, nullptr, 0};
+    const ZeroSpans zero = {{nullptr, nullptr, nullptr}, {0, 0, 0}};
+    return dispatch_k<256, true, false, false>(map, p, bits, counts, nullptr, nullptr, zero,
+                                               nullptr, none, s);
+}
+
 }  // namespace dol

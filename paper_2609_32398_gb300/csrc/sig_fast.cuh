@@ -1,5 +1,6 @@
-// Step 1, fast path (E in {32, 64, 128}, k in {1, 2, 4, 8}, 16-byte aligned
-// logits): Top-K signatures (Sec. 3.1.1, Eq. 1) with one token per lane.
+// Step 1, fast path (E in {32, 64, 128, 256}, k in {1, 2, 4, 8}, 16-byte
+// aligned logits; at E = 256 without the co-occurrence counts): Top-K
+// signatures (Sec. 3.1.1, Eq. 1) with one token per lane.
 //
 // A persistent CTA per SM owns a contiguous range of 32-token tiles.  One
 // producer warp streams each tile [32 tokens x E] into a ring of shared
@@ -43,11 +44,12 @@ template <int E>
 struct SigCfg {
     static constexpr int kBoxes = E / 32;
     static constexpr int kTileBytes = kBoxes * kBoxBytes;
-    static constexpr int kSlots = (E == 128) ? 11 : 16;
+    static constexpr int kSlots = (E == 256) ? 6 : (E == 128) ? 11 : 16;
     static constexpr int GS = (E >= 128) ? E / 16 : 4;  // experts per group
     static constexpr int NG = E / GS;                    // groups per row
-    // co-occurrence counters: row a holds columns (a & ~3) .. E-1
-    static constexpr int kCoocWords = cooc_row_offset<E>(E);
+    // co-occurrence counters: row a holds columns (a & ~3) .. E-1 (E <= 128;
+    // at E = 256 the kernel runs without them)
+    static constexpr int kCoocWords = E <= 128 ? cooc_row_offset<E>(E) : 0;
     static constexpr size_t kSmem = (size_t)kSlots * kTileBytes + 1024 + 2 * kSlots * 8 +
                                     kSlots * 4 + 32 + (size_t)kCoocWords * 4 + E * 4 +
                                     (size_t)kConsumers * E * 4;

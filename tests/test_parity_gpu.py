@@ -205,7 +205,8 @@ def test_host_entry_point_matches_device_path(dl):
     "T,E,k,L,gate,ties",
     [(1, 128, 8, 1, 0, False), (31, 32, 1, 2, 1, True), (97, 64, 2, 3, 0, True),
      (1000, 128, 4, 2, 1, False), (4096 + 33, 128, 8, 2, 0, True), (777, 32, 8, 1, 0, False),
-     (3000, 64, 8, 1, 1, True), (2048, 128, 1, 1, 0, True)])
+     (3000, 64, 8, 1, 1, True), (2048, 128, 1, 1, 0, True), (3000 + 5, 256, 8, 2, 0, True),
+     (777, 256, 1, 1, 1, False), (4096, 256, 4, 3, 0, True), (1000, 256, 2, 1, 0, False)])
 def test_fast_path_shapes(dl, T, E, k, L, gate, ties):
     z = workloads.random_logits(T, E, L=L, seed=T + 13 * E + k, ties=ties)
     out = gpu_run(dl, z, k, gate, grad_scale=3.0)
