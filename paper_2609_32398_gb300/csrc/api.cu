@@ -287,6 +287,30 @@ do_status forward_backward_impl(const float *logits, int64_t T, int32_t E, int32
         if (e == cudaSuccess && status_done) *status_done = status_out != nullptr;
         return from_cuda(e);
     }
+    if (!ra && dol::signatures_fast256_supported(logits, p) && aligned(bits, 16) &&
+        dol::loss_fast256_supported(p, logits, D, dlogits)) {
+        // E = 256: the fast selection (with the chosen experts), the Hamming
+        // matrix from the signatures, and the ALU loss kernel with D in
+        // shared-memory planes
+        const dol::WsLayout w = dol::ws_layout(p);
+        char *ws = static_cast<char *>(workspace);
+        int *done = reinterpret_cast<int *>(ws + w.done);
+        uint8_t *idx = reinterpret_cast<uint8_t *>(ws + w.idx);
+        int *status = reinterpret_cast<int *>(ws);
+        const dol::ZeroSpans zero = {{done, status_out, nullptr},
+                                     {(int64_t)p.L, status_out ? 1 : 0, 0}};
+        cudaError_t e = cudaMemsetAsync(counts, 0, sizeof(int) * (size_t)p.L * p.E, s);
+        if (e == cudaSuccess)
+            e = dol::launch_signatures_fast256(logits, p, bits, counts, idx, zero, status, s);
+        if (e == cudaSuccess) e = dol::launch_hamming(bits, p, D, s);
+        if (e == cudaSuccess)
+            e = dol::launch_loss_fast(logits, idx, D, counts, nullptr, p, gate, 1.0f, grad_scale,
+                                      loss, reinterpret_cast<long long *>(origin_do), dlogits,
+                                      reinterpret_cast<double *>(ws + w.partials), done, status,
+                                      status_out, s);
+        if (e == cudaSuccess && status_done) *status_done = status_out != nullptr;
+        return from_cuda(e);
+    }
     cudaError_t e = dol::launch_signatures(logits, p, bits, counts, s, route);
     if (e == cudaSuccess) e = dol::launch_hamming(bits, p, D, s);
     if (e == cudaSuccess)

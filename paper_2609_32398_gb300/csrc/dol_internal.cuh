@@ -96,10 +96,13 @@ cudaError_t launch_signatures(const float *logits, const Problem &p, uint32_t *b
                               const RouteOut &route = RouteOut{nullptr, nullptr, 0});
 cudaError_t launch_hamming(const uint32_t *bits, const Problem &p, int *D, cudaStream_t s);
 // The fast selection at E = 256 (k in {1, 2, 4, 8}, 16-byte aligned logits):
-// signatures and counts (counts zero on entry), no co-occurrence.
+// signatures and counts (counts zero on entry), no co-occurrence; idx (may be
+// null) the chosen experts of every token; zero: ranges cleared for the
+// kernels after it; status (may be null): the device status word.
 bool signatures_fast256_supported(const float *logits, const Problem &p);
 cudaError_t launch_signatures_fast256(const float *logits, const Problem &p, uint32_t *bits,
-                                      int *counts, cudaStream_t s);
+                                      int *counts, uint8_t *idx, const ZeroSpans &zero,
+                                      int *status, cudaStream_t s);
 cudaError_t launch_add_distances(const int *D, int *D_sum, int64_t n, cudaStream_t s);
 cudaError_t launch_hamming_accumulate(const uint32_t *bits, const Problem &p, int *D, cudaStream_t s);
 cudaError_t launch_origin_do(const int *D, const Problem &p, long long *origin_do, cudaStream_t s);
@@ -155,6 +158,9 @@ cudaError_t launch_router_signatures(const void *X, const void *Wr, int H, float
                                      uint32_t *cooc, const ZeroSpans &zero, int *status,
                                      cudaStream_t s);
 bool loss_fast_supported(const Problem &p, const float *logits, const int *D, const float *dlogits);
+// The E = 256 variant: counts given (D of the same tokens), T < 2^24.
+bool loss_fast256_supported(const Problem &p, const float *logits, const int *D,
+                            const float *dlogits);
 cudaError_t launch_idx_from_bits(const uint32_t *bits, const Problem &p, uint8_t *idx, int *zero_ptr,
                                  int zero_n, cudaStream_t s);
 // counts: when given, R_i = (E - 2k) n_i + T k (D local to these tokens) and

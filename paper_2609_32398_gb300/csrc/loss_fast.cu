@@ -1,5 +1,6 @@
-// Step 3, fast path (E in {32, 64, 128}, k in {1, 2, 4, 8}): the surrogate
-// DO-loss and its gradient (Sec. 3.1.3, Eq. do_loss; Eq. global_do scaling).
+// Step 3, fast path (E in {32, 64, 128, 256}, k in {1, 2, 4, 8}): the
+// surrogate DO-loss and its gradient (Sec. 3.1.3, Eq. do_loss; Eq. global_do
+// scaling).
 //
 // With R_i = sum_j D_ij, put D'_ij = D_ij off the diagonal and D'_ii = -R_i.
 // Then for the k experts S_t of token t
@@ -24,6 +25,15 @@
 //   softmax       e = exp(z - max), A = sum e w / sum e, dz = c e (w - A) / sum e
 // with c = grad_scale d_scale / (m^2 k).  A is summed per CTA in fp64 and the
 // last CTA of each problem adds the CTA partials in index order.
+//
+// At E = 256 an int32 D (256 KB) does not fit in shared memory: D is kept
+// there as a 16-bit low plane and an 8-bit high plane (192 KB; exact for the
+// matrix of the same tokens, whose entries are at most T < 2^24), with zeros
+// on the diagonal, and the -R_i of the k chosen experts are added to their
+// sums after the gather (R from the counts).  A row chunk of 4 entries is one
+// 8-byte and one 4-byte load; the low halves are summed per entry and the
+// high bytes in pairs of 16-bit fields, joined after the k rows.  One CTA of
+// 512 threads per SM.
 #include <climits>
 
 #include "dol_internal.cuh"
@@ -34,6 +44,13 @@ namespace {
 
 constexpr int kLossFastThreads = 256;
 constexpr int kLossFastWarps = kLossFastThreads / 32;
+// E = 256: one CTA per SM (the planes of D take 192 KB), with more warps
+constexpr int kLossPlaneThreads = 512;
+constexpr int kLossPlaneWarps = kLossPlaneThreads / 32;
+template <int E>
+constexpr int loss_fast_threads() { return E == 256 ? kLossPlaneThreads : kLossFastThreads; }
+template <int E>
+constexpr size_t loss_fast_smem() { return E == 256 ? (size_t)3 * E * E : sizeof(int) * E * E; }
 
 __device__ __forceinline__ float ex2_approx(float x) {
     float y;
@@ -99,15 +116,20 @@ struct LossArgs {
 };
 
 template <int E, int K, int kGate, bool kRFromCounts>
-__global__ void __launch_bounds__(kLossFastThreads, 3)
+__global__ void __launch_bounds__(loss_fast_threads<E>(), E == 256 ? 1 : 3)
 loss_fast_kernel(const LossArgs a) {
     constexpr int G = E / 16;    // lanes per token
     constexpr int TPW = 32 / G;  // tokens per warp pass
     constexpr int Q = E / 4;     // expert stride between a lane's chunks
-    extern __shared__ __align__(128) int sD[];  // [E][E]
+    constexpr bool kPlanes = E == 256;
+    constexpr int kWarps = loss_fast_threads<E>() / 32;
+    static_assert(!kPlanes || kRFromCounts, "the planes hold the matrix of the same tokens");
+    extern __shared__ __align__(128) int sD[];  // [E][E], or the two planes
+    uint16_t *sLo = reinterpret_cast<uint16_t *>(sD);             // [E][E] (planes)
+    uint8_t *sHi = reinterpret_cast<uint8_t *>(sD) + 2 * E * E;    // [E][E] (planes)
     __shared__ __align__(8) uint64_t bar;
-    __shared__ double s_part[kLossFastWarps];
-    __shared__ long long s_o[kLossFastWarps];
+    __shared__ double s_part[kWarps];
+    __shared__ long long s_o[kWarps];
     __shared__ long long s_r[E];
     __shared__ int s_last;
 
@@ -121,7 +143,7 @@ loss_fast_kernel(const LossArgs a) {
     const uint8_t *il = a.idx + (int64_t)layer * T * K;
     const int64_t t_begin = (int64_t)blockIdx.x * a.tokens_per_cta;
     const int64_t t_end = min64(T, t_begin + a.tokens_per_cta);
-    const int64_t stride = (int64_t)kLossFastWarps * TPW;
+    const int64_t stride = (int64_t)kWarps * TPW;
 
     pdl_trigger();  // the next kernel may be scheduled (it waits for this one to finish)
     if (threadIdx.x == 0) {
@@ -142,16 +164,39 @@ loss_fast_kernel(const LossArgs a) {
     __syncthreads();
     pdl_wait();  // D, idx and the cleared counters come from the previous kernels
     if (a.img_ok && __ldg(a.img_ok + layer) != 0) return;
-    if (threadIdx.x == 0) {
+    if (!kPlanes && threadIdx.x == 0) {
         mbar_arrive_expect_tx(&bar, (uint32_t)(sizeof(int) * E * E));
         bulk_load(sD, a.D + (int64_t)layer * E * E, (uint32_t)(sizeof(int) * E * E), &bar);
+    }
+    if constexpr (kPlanes) {
+        // four entries of a row per load: low halves and high bytes, the
+        // diagonal zero; an entry outside [0, 2^24) is reported
+        const int4 *src = reinterpret_cast<const int4 *>(a.D + (int64_t)layer * E * E);
+        int bad = 0;
+        for (int q = threadIdx.x; q < E * E / 4; q += blockDim.x) {
+            const int4 v = __ldg(src + q);
+            const int e0 = 4 * q, i = e0 / E, j0 = e0 % E;
+            int x[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                if (j0 + u == i) x[u] = 0;
+                bad |= (unsigned)x[u] >= (1u << 24);
+            }
+            *reinterpret_cast<uint2 *>(sLo + e0) =
+                make_uint2(((uint32_t)x[0] & 0xFFFFu) | ((uint32_t)x[1] << 16),
+                           ((uint32_t)x[2] & 0xFFFFu) | ((uint32_t)x[3] << 16));
+            *reinterpret_cast<uint32_t *>(sHi + e0) =
+                (((uint32_t)x[0] >> 16) & 0xFFu) | ((((uint32_t)x[1] >> 16) & 0xFFu) << 8) |
+                ((((uint32_t)x[2] >> 16) & 0xFFu) << 16) | ((((uint32_t)x[3] >> 16) & 0xFFu) << 24);
+        }
+        if (bad) atomicOr(a.status, kDevOverflow);
     }
     int js[K];
     {
         const int64_t t = tb + grp;
         load_idx<K>(il + ((t < t_end) ? t : t_begin) * K, js);
     }
-    const bool have_d = mbar_wait(&bar, 0, a.status);
+    const bool have_d = kPlanes || mbar_wait(&bar, 0, a.status);
     if (__syncthreads_or(!have_d)) return;
 
     if (kRFromCounts) {
@@ -160,7 +205,8 @@ loss_fast_kernel(const LossArgs a) {
             const long long n = a.counts[(int64_t)layer * E + i];
             const long long r = (long long)(E - 2 * K) * n + T * (long long)K;
             if (r > INT_MAX || r < 0) atomicOr(a.status, kDevOverflow);
-            sD[i * E + i] = -(int)r;
+            if (kPlanes) s_r[i] = r;
+            else sD[i * E + i] = -(int)r;
             if (a.n_zero && blockIdx.x == 0) a.n_zero[(int64_t)layer * E + i] = 0;
         }
     } else {
@@ -205,16 +251,60 @@ loss_fast_kernel(const LossArgs a) {
         int4 acc[4];
 #pragma unroll
         for (int c = 0; c < 4; ++c) acc[c] = make_int4(0, 0, 0, 0);
+        if constexpr (kPlanes) {
+            uint32_t hp[4][2];  // high bytes of entries (0, 2) and (1, 3), 16-bit fields
 #pragma unroll
-        for (int q = 0; q < K; ++q) {
-            const int *row = sD + js[q] * E + 4 * g;
+            for (int c = 0; c < 4; ++c) hp[c][0] = hp[c][1] = 0u;
+#pragma unroll
+            for (int q = 0; q < K; ++q) {
+                const int base = js[q] * E + 4 * g;
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    const uint2 lw = *reinterpret_cast<const uint2 *>(sLo + base + c * Q);
+                    const uint32_t hw = *reinterpret_cast<const uint32_t *>(sHi + base + c * Q);
+                    acc[c].x += (int)(lw.x & 0xFFFFu);
+                    acc[c].y += (int)(lw.x >> 16);
+                    acc[c].z += (int)(lw.y & 0xFFFFu);
+                    acc[c].w += (int)(lw.y >> 16);
+                    hp[c][0] += __byte_perm(hw, 0u, 0x4240);
+                    hp[c][1] += __byte_perm(hw, 0u, 0x4341);
+                }
+            }
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
-                const int4 d = *reinterpret_cast<const int4 *>(row + c * Q);
-                acc[c].x += d.x;
-                acc[c].y += d.y;
-                acc[c].z += d.z;
-                acc[c].w += d.w;
+                acc[c].x += (int)((hp[c][0] & 0xFFFFu) << 16);
+                acc[c].z += (int)(hp[c][0] & 0xFFFF0000u);
+                acc[c].y += (int)((hp[c][1] & 0xFFFFu) << 16);
+                acc[c].w += (int)(hp[c][1] & 0xFFFF0000u);
+            }
+            // the diagonal of D': -R_j in the sum of each chosen expert j
+#pragma unroll
+            for (int q = 0; q < K; ++q) {
+                const int j = js[q];
+                if (((j & (Q - 1)) >> 2) != g) continue;
+                const int rj = (int)s_r[j];
+                const int cj = j / Q, ej = j & 3;
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    if (c != cj) continue;
+                    acc[c].x -= ej == 0 ? rj : 0;
+                    acc[c].y -= ej == 1 ? rj : 0;
+                    acc[c].z -= ej == 2 ? rj : 0;
+                    acc[c].w -= ej == 3 ? rj : 0;
+                }
+            }
+        } else {
+#pragma unroll
+            for (int q = 0; q < K; ++q) {
+                const int *row = sD + js[q] * E + 4 * g;
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    const int4 d = *reinterpret_cast<const int4 *>(row + c * Q);
+                    acc[c].x += d.x;
+                    acc[c].y += d.y;
+                    acc[c].z += d.z;
+                    acc[c].w += d.w;
+                }
             }
         }
         float w[16], zz[16], gv[16];
@@ -288,7 +378,7 @@ loss_fast_kernel(const LossArgs a) {
     __syncthreads();
     if (threadIdx.x == 0) {
         double sum = 0.0;
-        for (int q = 0; q < kLossFastWarps; ++q) sum += s_part[q];
+        for (int q = 0; q < kWarps; ++q) sum += s_part[q];
         a.partials[(int64_t)layer * P + blockIdx.x] = sum;
         __threadfence();
         s_last = (atomicAdd(&a.done[layer], 1) == P - 1);
@@ -310,7 +400,8 @@ loss_fast_kernel(const LossArgs a) {
         for (int e = threadIdx.x; e < E * E; e += blockDim.x) {
             const int i = e / E, j = e - (e / E) * E;
             if (i != j) {
-                const long long d = sD[e];
+                const long long d =
+                    kPlanes ? (long long)sLo[e] | ((long long)sHi[e] << 16) : (long long)sD[e];
                 o += d * d;
             }
         }
@@ -320,7 +411,7 @@ loss_fast_kernel(const LossArgs a) {
         __syncthreads();
         if (threadIdx.x == 0) {
             long long sum = 0;
-            for (int q = 0; q < kLossFastWarps; ++q) sum += s_o[q];
+            for (int q = 0; q < kWarps; ++q) sum += s_o[q];
             a.origin_do[layer] = sum;
         }
     }
@@ -383,13 +474,13 @@ idx_from_bits_kernel(const uint32_t *__restrict__ bits, int64_t T, int64_t W, in
 
 template <int E, int K, bool kRFromCounts>
 cudaError_t run_loss_fast(const LossArgs &args, int gate, int P, const Problem &p, cudaStream_t s) {
-    const size_t smem = sizeof(int) * E * E;
+    const size_t smem = loss_fast_smem<E>();
     cudaError_t e = ensure_smem_limit<loss_fast_kernel<E, K, 0, kRFromCounts>>(smem);
     if (e == cudaSuccess) e = ensure_smem_limit<loss_fast_kernel<E, K, 1, kRFromCounts>>(smem);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)P, (unsigned)p.L);
-    cfg.blockDim = dim3(kLossFastThreads);
+    cfg.blockDim = dim3(loss_fast_threads<E>());
     cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
@@ -432,12 +523,24 @@ bool loss_fast_supported(const Problem &p, const float *logits, const int *D, co
            (dlogits == nullptr || reinterpret_cast<uintptr_t>(dlogits) % 16 == 0);
 }
 
+// The E = 256 variant (the matrix of the same tokens, with counts): T < 2^24
+// keeps every entry of D within the 24 bits of its shared-memory planes.
+bool loss_fast256_supported(const Problem &p, const float *logits, const int *D,
+                            const float *dlogits) {
+    const bool k_ok = p.k == 1 || p.k == 2 || p.k == 4 || p.k == 8;
+    return p.E == 256 && k_ok && p.T < (int64_t)(1 << 24) &&
+           reinterpret_cast<uintptr_t>(logits) % 16 == 0 &&
+           reinterpret_cast<uintptr_t>(D) % 16 == 0 &&
+           (dlogits == nullptr || reinterpret_cast<uintptr_t>(dlogits) % 16 == 0);
+}
+
 // CTAs per problem of the fast loss kernel and the tokens each one takes.
 void loss_fast_grid(const Problem &p, int *P, int *tokens_per_cta) {
     int dev = 0, sms = 148;
     if (cudaGetDevice(&dev) == cudaSuccess)
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    int64_t want = (int64_t)sms * 3 / p.L;  // three CTAs fit on an SM: one wave
+    // one wave: three CTAs fit on an SM, one at E = 256
+    int64_t want = (int64_t)sms * (p.E == 256 ? 1 : 3) / p.L;
     if (want < 1) want = 1;
     int64_t tpc = (p.T + want - 1) / want;
     tpc = (tpc + 31) / 32 * 32;
@@ -494,8 +597,10 @@ cudaError_t launch_loss_fast(const float *logits, const uint8_t *idx, const int 
     if (counts) {
         if (p.E == 32) return dispatch_loss_k<32, true>(args, gate, P, p, s);
         if (p.E == 64) return dispatch_loss_k<64, true>(args, gate, P, p, s);
+        if (p.E == 256) return dispatch_loss_k<256, true>(args, gate, P, p, s);
         return dispatch_loss_k<128, true>(args, gate, P, p, s);
     }
+    if (p.E == 256) return cudaErrorInvalidValue;  // the planes need the counts' R
     if (p.E == 32) return dispatch_loss_k<32, false>(args, gate, P, p, s);
     if (p.E == 64) return dispatch_loss_k<64, false>(args, gate, P, p, s);
     return dispatch_loss_k<128, false>(args, gate, P, p, s);

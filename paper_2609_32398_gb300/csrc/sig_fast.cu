@@ -53,14 +53,14 @@ bool signatures_fast256_supported(const float *logits, const Problem &p) {
 }
 
 cudaError_t launch_signatures_fast256(const float *logits, const Problem &p, uint32_t *bits,
-                                      int *counts, cudaStream_t s) {
+                                      int *counts, uint8_t *idx, const ZeroSpans &zero,
+                                      int *status, cudaStream_t s) {
     CUtensorMap map;
     if (!encode_tensor_map_2d_f32(&map, logits, (uint64_t)p.L * p.T, (uint64_t)p.E, 32))
         return cudaErrorInvalidValue;
     const RouteOut none = {nullptr, nullptr, 0};
-    const ZeroSpans zero = {{nullptr, nullptr, nullptr}, {0, 0, 0}};
-    return dispatch_k<256, true, false, false>(map, p, bits, counts, nullptr, nullptr, zero,
-                                               nullptr, none, s);
+    return dispatch_k<256, true, false, false>(map, p, bits, counts, idx, nullptr, zero, status,
+                                               none, s);
 }
 
 }  // namespace dol

@@ -132,8 +132,10 @@ cudaError_t launch_signatures(const float *logits, const Problem &p, uint32_t *b
                               cudaStream_t s, const RouteOut &route) {
     cudaError_t e = cudaMemsetAsync(counts, 0, sizeof(int) * (size_t)p.L * p.E, s);
     if (e != cudaSuccess) return e;
-    if (!route.ids && signatures_fast256_supported(logits, p))
-        return launch_signatures_fast256(logits, p, bits, counts, s);
+    if (!route.ids && signatures_fast256_supported(logits, p)) {
+        const ZeroSpans none = {{nullptr, nullptr, nullptr}, {0, 0, 0}};
+        return launch_signatures_fast256(logits, p, bits, counts, nullptr, none, nullptr, s);
+    }
     const int r = (p.E + 31) / 32;
     if (r <= 1) return run_generic<1>(logits, p, bits, counts, route, s);
     if (r <= 2) return run_generic<2>(logits, p, bits, counts, route, s);
