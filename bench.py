@@ -415,6 +415,13 @@ def run_ours(args, rank, world, local):
                 dl.routed_backward(sets[i % N_SETS][0], route.expert_ids, gq, k, w.gate, 1.0,
                                    out=sets[i % N_SETS][1])
             ws = sets[0][1].workspace
+        elif args.quick_path == "hamming":
+            bits0, _ = dl.signatures(sets[0][0], k)
+            Dh = torch.empty(L, E, E, dtype=torch.int32, device=dev)
+
+            def call(i):
+                dl.pairwise_hamming(bits0, T, Dh)
+            ws = sets[0][1].workspace
         elif args.quick_path == "route_bwd":
             route = dl.routing(sets[0][0], k, w.gate)
             gq = torch.randn(L, T, k, device=dev)
@@ -891,11 +898,12 @@ def main():
     ap.add_argument("--quick", action="store_true",
                     help="run warmup+steps plain steps and exit (for profilers)")
     ap.add_argument("--quick-path", choices=["loss", "routing", "routed", "router", "route_bwd",
-                                             "split"],
+                                             "split", "hamming"],
                     default="loss",
                     help="entry point of --quick: do_forward_backward, do_routing, "
                          "do_forward_backward_routed, do_router_forward_backward, "
-                         "do_route_backward or do_routed_forward + do_routed_backward")
+                         "do_route_backward, do_routed_forward + do_routed_backward or "
+                         "do_pairwise_hamming")
     args = ap.parse_args()
     if args.impl == "reference":
         rank = int(os.environ.get("RANK", "0"))
