@@ -89,8 +89,10 @@ do_status do_signatures(const float *logits, int64_t T, int32_t E, int32_t k, in
                         uint32_t *bits, int32_t *counts, void *stream);
 
 /* Step 2 (Sec. 3.1.3, Eq. gij_cij: G_ij = ||F_i - F_j||_1).
- * Reads bits [L][E][W]; writes D [L][E][E], the exact number of tokens on
- * which experts i and j disagree. */
+ * Reads bits [L][E][W] (4-byte aligned; the bits past T in the last word
+ * zero, as do_signatures writes them); writes D [L][E][E], the exact number
+ * of tokens on which experts i and j disagree, every entry once (no
+ * clearing needed).  Uses thread-block clusters of up to 8 CTAs. */
 do_status do_pairwise_hamming(const uint32_t *bits, int64_t T, int32_t E, int32_t L,
                               int32_t *D, void *stream);
 
@@ -145,8 +147,10 @@ do_status do_loss_fwd_bwd(const float *logits, const uint32_t *bits, const int32
  * With E = 128, the sigmoid-normalised gate, k in {1, 2, 4, 8}, T <= 66052
  * and dlogits given, the gradient pass computes V = F D' on the tensor cores
  * (F the one-hot selections, D' = D with -R on the diagonal); elsewhere it
- * gathers rows of D' on the ALU (as do_loss_fwd_bwd always does).  The two
- * agree within the stated tolerances. */
+ * gathers rows of D' on the ALU (as do_loss_fwd_bwd always does; at E = 256,
+ * k in {1, 2, 4, 8}, T < 2^24 and 16-byte aligned logits, D and dlogits with
+ * D held in 24-bit shared-memory planes).  The two agree within the stated
+ * tolerances. */
 do_status do_forward_backward(const float *logits, int64_t T, int32_t E, int32_t k, int32_t L,
                               int32_t gate, float grad_scale, uint32_t *bits, int32_t *counts,
                               int32_t *D, float *loss, int64_t *origin_do, float *dlogits,
@@ -207,12 +211,18 @@ size_t do_routing_workspace_size(int64_t T, int32_t E, int32_t k, int32_t L);
  * it wrote.  With d_scale = 1, D is the forward half's matrix; otherwise D
  * is a matrix summed over data-parallel ranks or micro-batches that include
  * these tokens (Eq. global_do, d_scale = 1 / their number) and m stays T.
- * With d_scale = 1, E = 128, the sigmoid-normalised gate, k in {1, 2, 4, 8},
- * T <= 66052 and 16-byte aligned logits, D, bits, dlogits, expert_ids and
- * grad_combine, the tensor-core loss kernel runs and adds the routing
- * gradient in its epilogue (one launch); elsewhere the ALU loss kernels run
- * and a second kernel adds it.  The result agrees with do_loss_fwd_bwd's
- * dlogits plus do_route_backward's within the sum of their tolerances.
+ * With E = 128, the sigmoid-normalised gate, k in {1, 2, 4, 8} and 16-byte
+ * aligned logits, D, bits, dlogits, expert_ids and grad_combine, the
+ * tensor-core loss kernel runs and adds the routing gradient in its
+ * epilogue: with d_scale = 1 (and T <= 66052) from the image of D' the
+ * forward half left; otherwise a kernel first builds the image of the given
+ * matrix and checks, per problem, that its two fp16 pieces hold it exactly
+ * (0 <= D_ij < 2^22 off the diagonal, D_ii = 0, row sums below 2^23), and
+ * the problems that fail the check go to the ALU loss kernel and the
+ * routing-gradient kernel instead.  Elsewhere the ALU loss kernels run and a
+ * second kernel adds the routing gradient.  The result agrees with
+ * do_loss_fwd_bwd's dlogits plus do_route_backward's within the sum of their
+ * tolerances.
  *
  * Both take the same workspace (do_routed_workspace_size bytes, 256-byte
  * aligned, zero-filled before its first use): the forward half leaves in it
