@@ -204,7 +204,8 @@ hamming_kernel(const uint32_t *__restrict__ bits, int E, int64_t W, int nside, i
     }
     if (active) s_part[tile * 16 + q] = v[0];
     cluster_sync();
-    // CTA `rank` adds the C partial sums of entries [rank, +per_e) in rank order
+    // CTA `rank` adds, in rank order, the C partial sums of the entries
+    // rank * per_e .. (rank + 1) * per_e - 1 of the block
     const int per_e = kHTiles * 16 / C;
     for (int e = (int)rank * per_e + threadIdx.x; e < ((int)rank + 1) * per_e; e += kHThreads) {
         const int tl = e >> 4, idx = e & 15;
@@ -249,15 +250,14 @@ cudaError_t run_hamming(const uint32_t *bits, const Problem &p, int *D, int accu
     int sms = 0, per_sm = 0;
     cudaError_t e = hamming_slots(&sms, &per_sm);
     if (e != cudaSuccess) return e;
-    if (e == cudaSuccess) e = ensure_smem_limit<hamming_kernel>(kHSmem);
+    e = ensure_smem_limit<hamming_kernel>(kHSmem);
     if (e != cudaSuccess) return e;
     // split the words over a cluster while the units leave resident slots idle
     const int64_t slots = (int64_t)sms * per_sm;
     int C = 1;
     while (C < kHMaxCluster && units * p.L * C * 2 <= slots && C * 2 <= nst) C *= 2;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(units * C), 1u, 1u);
-    cfg.gridDim.y = (unsigned)p.L;
+    cfg.gridDim = dim3((unsigned)(units * C), (unsigned)p.L);
     cfg.blockDim = dim3(kHThreads);
     cfg.dynamicSmemBytes = kHSmem;
     cfg.stream = s;
