@@ -43,10 +43,8 @@ namespace dol {
 namespace {
 
 constexpr int kLossFastThreads = 256;
-constexpr int kLossFastWarps = kLossFastThreads / 32;
 // E = 256: one CTA per SM (the planes of D take 192 KB), with more warps
 constexpr int kLossPlaneThreads = 512;
-constexpr int kLossPlaneWarps = kLossPlaneThreads / 32;
 template <int E>
 constexpr int loss_fast_threads() { return E == 256 ? kLossPlaneThreads : kLossFastThreads; }
 template <int E>
